@@ -1,0 +1,260 @@
+/*
+ * fademem_oracle.c -- plain, slow, fp64 CPU oracle of FadeMem
+ * (arxiv 2606.10671, "FadeMem: Distance-Aware Memory Consolidation for
+ * Autoregressive Video Diffusion").
+ *
+ * TEST INFRASTRUCTURE ONLY.  The test-suite, the smoke check and the CPU
+ * baseline leg of the benchmark load this library; the CUDA library never
+ * includes, links or calls it, and this file includes nothing of the CUDA
+ * library.  Every result here is computed in IEEE double precision.
+ *
+ * What it computes
+ *   1. The online memory update of Algorithm S1 (supplementary Sec. S1), one
+ *      generation unit (one latent frame, Sec. S4) per call:
+ *        - append (K_t, V_t, mu = t, s = 1)                (Sec. 3.3, "insertion")
+ *        - if more than M entries, score every adjacent pair except the one
+ *          holding the newest entry by g_i = |u(t-mu_{i+1}) - u(t-mu_i)|,
+ *          u(d) = d^beta                     (Sec. 3.3, "distance-aware scheduling")
+ *        - j = argmin_i g_i
+ *        - s_new = s_j + s_{j+1}; if the pair holds the first-frame anchor the
+ *          result keeps the anchor's K/V and mu = 0 (Sec. 3.3, "boundary
+ *          handling"; Algorithm S1), otherwise mu_new is the span-weighted
+ *          centre and the K/V blocks are merged by the operator (Sec. 3.3,
+ *          "consolidation operator", square-root span weights by default;
+ *          Table 2 for the alternatives)
+ *        - the result replaces the pair.
+ *   2. Attention of query tokens over every token of every memory entry,
+ *      per head: out = softmax(scale * q K^T) V (the backbone attention whose
+ *      context the memory supplies, Sec. 3.3 last paragraph, Sec. 4.1).
+ *
+ * Readings where the paper is silent (each one also listed in the design notes):
+ *   - frames are numbered from t = 0, so the anchor's own centre is mu = 0;
+ *   - ties in the argmin go to the lowest pair index (the oldest pair);
+ *   - the anchor is entry 0; its pair is j == 0;
+ *   - storage slots: the paper has none.  To check a device slot table the
+ *     oracle also keeps one: the merged entry keeps the slot of m_j, and the
+ *     new entry takes the slot freed by m_{j+1} (or slot count-1 when no
+ *     merge happens).  This never changes what is computed.
+ *   - "Select Nearest" keeps the block of the entry nearer to the current step
+ *     (m_{j+1}, the smaller distance d).
+ *
+ * Layout of a K or V block: elems_per_block doubles, in the caller's order.
+ * For attention the order must be [token][head][dim] (tokens x heads x dim).
+ * Merges are elementwise, so a caller may also pass any subset of coordinates
+ * (e.g. a fixed sample), and the oracle's values at those coordinates are
+ * exactly those of the full computation.
+ */
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+enum { OP_WEIGHTED = 0, OP_AVERAGE = 1, OP_SELECT_NEAREST = 2, OP_MAX_POOL = 3 };
+
+struct entry {
+    int slot;           /* storage slot (reading: slot policy above) */
+    long long first;    /* first generation unit summarised */
+    long long span;     /* s: number of units summarised */
+    double mu;          /* temporal centre */
+    double *K, *V;      /* representative blocks */
+};
+
+typedef struct oracle_memory {
+    int M;               /* entry budget */
+    double beta;         /* warp exponent, 0 < beta <= 1 */
+    int anchor;          /* first-frame global anchor on/off */
+    int op;              /* consolidation operator */
+    long long elems;     /* doubles per K (or V) block */
+    long long t_next;    /* index of the next generation unit */
+    int count;           /* |M_t| */
+    struct entry *e;     /* e[0..count-1], temporal order; room for M+1 */
+    /* record of the latest update, for tests */
+    int last_j;          /* merged pair index, -1 if none */
+    double last_margin;  /* (g_second - g_min) / g_second, +inf if < 2 pairs */
+    double last_gmin;
+} oracle_memory;
+
+oracle_memory *oracle_create(int M, double beta, int anchor, int op, long long elems)
+{
+    if (M < 2 || !(beta > 0.0 && beta <= 1.0) || op < 0 || op > 3 || elems < 0) return NULL;
+    oracle_memory *m = (oracle_memory *)calloc(1, sizeof(*m));
+    if (!m) return NULL;
+    m->M = M; m->beta = beta; m->anchor = anchor ? 1 : 0; m->op = op; m->elems = elems;
+    m->e = (struct entry *)calloc((size_t)M + 1, sizeof(struct entry));
+    if (!m->e) { free(m); return NULL; }
+    m->last_j = -1;
+    return m;
+}
+
+void oracle_destroy(oracle_memory *m)
+{
+    if (!m) return;
+    for (int i = 0; i < m->count; ++i) { free(m->e[i].K); free(m->e[i].V); }
+    free(m->e);
+    free(m);
+}
+
+static double warp_u(double d, double beta) { return pow(d, beta); }   /* u(d) = d^beta */
+
+/* One update of Algorithm S1.  K_t, V_t: the new unit's blocks (elems doubles
+ * each; may be NULL when elems == 0, i.e. schedule-only runs).  Returns 0. */
+int oracle_insert(oracle_memory *m, const double *K_t, const double *V_t)
+{
+    const long long t = m->t_next++;
+    const size_t bytes = (size_t)m->elems * sizeof(double);
+
+    /* Append (K_t, V_t, t, 1). */
+    struct entry *nw = &m->e[m->count];
+    nw->first = t; nw->span = 1; nw->mu = (double)t;
+    nw->K = (double *)malloc(bytes ? bytes : 1);
+    nw->V = (double *)malloc(bytes ? bytes : 1);
+    if (bytes) { memcpy(nw->K, K_t, bytes); memcpy(nw->V, V_t, bytes); }
+    m->count += 1;
+    m->last_j = -1; m->last_margin = INFINITY; m->last_gmin = NAN;
+
+    /* |M_t| <= M: simply appended; it takes the next free slot. */
+    if (m->count <= m->M) { nw->slot = m->count - 1; return 0; }
+
+    /* Score every adjacent pair (i, i+1) except the pair holding the newest
+     * entry, which is (count-2, count-1). */
+    const int npairs = m->count - 2;
+    int j = 0;
+    double gmin = INFINITY, gsecond = INFINITY;
+    for (int i = 0; i < npairs; ++i) {
+        const double d_i = (double)t - m->e[i].mu;
+        const double d_i1 = (double)t - m->e[i + 1].mu;
+        const double g = fabs(warp_u(d_i1, m->beta) - warp_u(d_i, m->beta));
+        if (g < gmin) { gsecond = gmin; gmin = g; j = i; }       /* strict: lowest index wins ties */
+        else if (g < gsecond) { gsecond = g; }
+    }
+    m->last_j = j; m->last_gmin = gmin;
+    m->last_margin = (npairs >= 2) ? (gsecond - gmin) / gsecond : INFINITY;
+
+    struct entry *a = &m->e[j], *b = &m->e[j + 1];
+    const long long s_j = a->span, s_j1 = b->span;
+    const long long s_new = s_j + s_j1;
+    double mu_new;
+
+    if (m->anchor && j == 0) {
+        /* Pair holds the first-frame anchor: keep its blocks, mu = 0. */
+        mu_new = 0.0;
+    } else {
+        mu_new = ((double)s_j * a->mu + (double)s_j1 * b->mu) / (double)s_new;
+        double w_j, w_j1;
+        switch (m->op) {
+        case OP_AVERAGE:        w_j = 0.5; w_j1 = 0.5; break;
+        case OP_SELECT_NEAREST: w_j = 0.0; w_j1 = 1.0; break;
+        default:                w_j = sqrt((double)s_j) / (sqrt((double)s_j) + sqrt((double)s_j1));
+                                w_j1 = 1.0 - w_j; break;
+        }
+        for (long long k = 0; k < m->elems; ++k) {
+            if (m->op == OP_MAX_POOL) {
+                a->K[k] = fmax(a->K[k], b->K[k]);
+                a->V[k] = fmax(a->V[k], b->V[k]);
+            } else {
+                a->K[k] = w_j * a->K[k] + w_j1 * b->K[k];
+                a->V[k] = w_j * a->V[k] + w_j1 * b->V[k];
+            }
+        }
+    }
+    a->span = s_new;
+    a->mu = mu_new;
+    /* a->first and a->slot are kept (the result keeps m_j's slot). */
+
+    /* Remove m_{j+1}; the newest entry takes its slot. */
+    const int freed_slot = b->slot;
+    free(b->K); free(b->V);
+    for (int i = j + 1; i < m->count - 1; ++i) m->e[i] = m->e[i + 1];
+    m->count -= 1;
+    m->e[m->count - 1].slot = freed_slot;
+    return 0;
+}
+
+int oracle_count(const oracle_memory *m) { return m->count; }
+long long oracle_frames(const oracle_memory *m) { return m->t_next; }
+int oracle_last_pair(const oracle_memory *m) { return m->last_j; }
+double oracle_last_margin(const oracle_memory *m) { return m->last_margin; }
+double oracle_last_gmin(const oracle_memory *m) { return m->last_gmin; }
+
+void oracle_entries(const oracle_memory *m, int *slot, long long *first, long long *span, double *mu)
+{
+    for (int i = 0; i < m->count; ++i) {
+        if (slot) slot[i] = m->e[i].slot;
+        if (first) first[i] = m->e[i].first;
+        if (span) span[i] = m->e[i].span;
+        if (mu) mu[i] = m->e[i].mu;
+    }
+}
+
+/* Copy entry i's K and V blocks out (elems doubles each). */
+int oracle_entry_kv(const oracle_memory *m, int i, double *K, double *V)
+{
+    if (i < 0 || i >= m->count) return -1;
+    const size_t bytes = (size_t)m->elems * sizeof(double);
+    if (K) memcpy(K, m->e[i].K, bytes);
+    if (V) memcpy(V, m->e[i].V, bytes);
+    return 0;
+}
+
+/* Attention of Lq query tokens over every token of every entry.
+ * Q, out: [Lq][H][D].  Entry blocks: [tokens][H][D] with tokens*H*D == elems.
+ * For each query row and head: logits l_k = scale * <q, k_k> over all
+ * count*tokens keys, p = softmax(l) (max-subtracted), out = sum_k p_k v_k. */
+int oracle_attend(const oracle_memory *m, int tokens, int H, int D,
+                  const double *Q, long long Lq, double scale, double *out)
+{
+    if ((long long)tokens * H * D != m->elems || m->count == 0) return -1;
+    const long long Lk = (long long)m->count * tokens;
+    int failed = 0;
+#pragma omp parallel
+    {
+        double *logit = (double *)malloc((size_t)Lk * sizeof(double));
+        if (!logit) {
+#pragma omp atomic write
+            failed = 1;
+        }
+#pragma omp for collapse(2) schedule(dynamic, 4)
+        for (long long q = 0; q < Lq; ++q) {
+            for (int h = 0; h < H; ++h) {
+                if (!logit) continue;
+                const double *qv = Q + ((size_t)q * H + h) * D;
+                double mx = -INFINITY;
+                long long k = 0;
+                for (int e = 0; e < m->count; ++e) {
+                    for (int n = 0; n < tokens; ++n, ++k) {
+                        const double *kv = m->e[e].K + ((size_t)n * H + h) * D;
+                        double dot = 0.0;
+                        for (int d = 0; d < D; ++d) dot += qv[d] * kv[d];
+                        logit[k] = scale * dot;
+                        if (logit[k] > mx) mx = logit[k];
+                    }
+                }
+                double Z = 0.0;
+                for (k = 0; k < Lk; ++k) { logit[k] = exp(logit[k] - mx); Z += logit[k]; }
+                double *o = out + ((size_t)q * H + h) * D;
+                for (int d = 0; d < D; ++d) o[d] = 0.0;
+                k = 0;
+                for (int e = 0; e < m->count; ++e) {
+                    for (int n = 0; n < tokens; ++n, ++k) {
+                        const double *vv = m->e[e].V + ((size_t)n * H + h) * D;
+                        const double p = logit[k] / Z;
+                        for (int d = 0; d < D; ++d) o[d] += p * vv[d];
+                    }
+                }
+            }
+        }
+        free(logit);
+    }
+    return failed ? -2 : 0;
+}
+
+int oracle_num_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}

@@ -1,0 +1,26 @@
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a); runs the CUDA library")
+    config.addinivalue_line("markers", "slow: long CPU-side check")
+
+
+@pytest.fixture(scope="session")
+def oracle_lib():
+    from oracle import build_oracle
+    return build_oracle()
+
+
+@pytest.fixture(scope="session")
+def cuda_lib():
+    """The CUDA library, built in-tree if missing (nvcc cross-compiles without a GPU)."""
+    from paper_2606_10671_gb300 import build
+    return build.build_library()
