@@ -1,0 +1,360 @@
+#!/usr/bin/env python3
+"""Benchmark of FadeMem's per-segment memory step on GB300 (one JSON line).
+
+Workload (Wan2.1-1.3B shaped, one layer, bf16): 12 heads, head_dim 128, 1560
+tokens per latent frame, 3-frame segments (4680 query tokens), budget 21
+entries, beta 0.3, first-frame anchor on, synthetic AR(1) K/V (rho 0.9) and
+N(0,1) queries.  The memory is first brought to steady state (21 entries, 3
+merges per segment).  One step = insert the segment's 3 frames + device
+schedule + fused consolidation + attention of the 4680 queries over the 21
+consolidated entries (32,760 keys per head).
+
+Metric: query tokens per second per layer over (attend + consolidate) time.
+`value` times the device-resident step with CUDA events, L2 flushed (256 MiB
+write) before every step and excluded from the step time.  `e2e` times the
+same step through the C ABI with pinned host buffers: host->device copy of
+K, V and Q, the three calls, device->host copy of the output.
+
+--impl reference times the fp64 CPU oracle on this machine's cores on a
+bounded sample of the same workload (see cpu_baseline).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+H, D, N, F, M, BETA = 12, 128, 1560, 3, 21, 0.3
+LQ = F * N
+WORKLOAD = "wan2.1-1.3b-shaped single layer: H=12 D=128 N=1560 frames/segment=3 Lq=4680 M=21 beta=0.3 bf16"
+METRIC = "query tokens/s per layer (attend+consolidate)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            p = json.load(fh)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        try:
+            for ln in open(self.path):
+                parts = [x.strip() for x in ln.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        except Exception:
+            pass
+        finally:
+            try:
+                os.unlink(self.path)
+            except Exception:
+                pass
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        busy = sorted(sm)[len(sm) // 4:] if sm else []  # samples under load (drop idle ramp)
+        return {"sm_mhz": statistics.median(busy) if busy else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _segment_inputs(seed, n_sets, device):
+    """n_sets distinct (K, V, Q) segment inputs, AR(1) K/V across the sets' frames."""
+    from synth import KIND_K, KIND_V, DeviceAR1, device_queries
+    gk = DeviceAR1((N, H, D), seed, KIND_K, 0, device=device)
+    gv = DeviceAR1((N, H, D), seed, KIND_V, 0, device=device)
+    sets = []
+    for s in range(n_sets):
+        K = torch.stack([gk.next() for _ in range(F)]).contiguous()
+        V = torch.stack([gv.next() for _ in range(F)]).contiguous()
+        Q = device_queries((LQ, H, D), seed, 0, s, device=device)
+        sets.append((K, V, Q))
+    return sets
+
+
+def run_cuda(args):
+    from paper_2606_10671_gb300 import FadeMem
+    from paper_2606_10671_gb300 import build as _b
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    _b.build_library()
+
+    mem = FadeMem(M, H, D, N, num_layers=1, beta=BETA, anchor=True, dtype=torch.bfloat16, device=dev)
+    n_sets = 4
+    sets = _segment_inputs(1000 + rank, n_sets, dev)
+    out = torch.empty((LQ, H, D), dtype=torch.bfloat16, device=dev)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    # Steady state: 8 segments of 3 frames fill the 21-entry budget and start merging.
+    for s in range(8):
+        K, V, _ = sets[s % n_sets]
+        mem.insert(0, K, V)
+        mem.consolidate()
+
+    def step(i):
+        K, V, Q = sets[i % n_sets]
+        mem.insert(0, K, V)
+        mem.consolidate()
+        return Q
+
+    for i in range(args.warmup):
+        Q = step(i)
+        mem.attend(0, Q, out)
+    torch.cuda.synchronize()
+    mem.device_status()
+
+    # algorithmic bytes of the consolidation: every plan source read once, every changed slot written once
+    block_bytes = 2 * N * H * D * 2  # K + V of one entry of one layer, bf16
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    plan_blocks = []
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    region0 = torch.cuda.Event(enable_timing=True)
+    region1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(torch.cuda.current_device() if "CUDA_VISIBLE_DEVICES" not in os.environ else local) as clk:
+        region0.record(stream)
+        for i in range(args.steps):
+            flush.zero_()
+            e0, e1, e2 = ev[i]
+            e0.record(stream)
+            Q = step(args.warmup + i)
+            e1.record(stream)
+            mem.attend(0, Q, out)
+            e2.record(stream)
+        region1.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    clocks = clk.summary()
+    t_cons = [ev[i][0].elapsed_time(ev[i][1]) for i in range(args.steps)]
+    t_attn = [ev[i][1].elapsed_time(ev[i][2]) for i in range(args.steps)]
+    ns, nd, _ = mem.last_plan()
+    plan_blocks.append(ns + nd)
+    mem.device_status()
+    step_ms = (sum(t_cons) + sum(t_attn)) / args.steps
+    if ws > 1:
+        t = torch.tensor([step_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        step_ms = float(t.item())
+    value = ws * LQ / (step_ms / 1e3)
+
+    hbm_peak, bf16_peak, peak_kind = _peaks()
+    attn_ms = statistics.mean(t_attn)
+    cons_ms = statistics.mean(t_cons)
+    Lk = M * N
+    flops = 4.0 * LQ * Lk * H * D
+    attn_tflops = flops / (attn_ms / 1e3) / 1e12
+    cons_bytes = plan_blocks[-1] * block_bytes
+    cons_gbs = cons_bytes / (cons_ms / 1e3) / 1e9
+
+    # End to end through the C ABI with host buffers.
+    hK = [s[0].cpu().pin_memory() for s in sets]
+    hV = [s[1].cpu().pin_memory() for s in sets]
+    hQ = [s[2].cpu().pin_memory() for s in sets]
+    hO = torch.empty((LQ, H, D), dtype=torch.bfloat16).pin_memory()
+    dK = torch.empty_like(sets[0][0])
+    dV = torch.empty_like(sets[0][1])
+    dQ = torch.empty_like(sets[0][2])
+    e2e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        j = i % n_sets
+        flush.zero_()
+        a, b = e2e_ev[i]
+        a.record(stream)
+        dK.copy_(hK[j], non_blocking=True)
+        dV.copy_(hV[j], non_blocking=True)
+        dQ.copy_(hQ[j], non_blocking=True)
+        mem.insert(0, dK, dV)
+        mem.consolidate()
+        mem.attend(0, dQ, out)
+        hO.copy_(out, non_blocking=True)
+        b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
+    if ws > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    h2d = sum(x.numel() * x.element_size() for x in (hK[0], hV[0], hQ[0]))
+    d2h = hO.numel() * hO.element_size()
+    mem.device_status()
+
+    line = {
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": "tokens/s",
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(step_ms, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (AR(1) K/V rho=0.9, N(0,1) Q; no model weights)",
+        "config": {"workload": WORKLOAD, "steady_state_entries": M, "keys_per_head": Lk,
+                   "l2": "flushed before every step (256 MiB write), flush excluded from step time",
+                   "parallelism": f"replicas x{ws} (one independent memory per GPU)"},
+        "gpu_launches": 3 * args.steps,
+        "roofline": {"bound": "tensor", "kernel": "attend_tc_kernel", "achieved": round(attn_tflops, 1),
+                     "peak": bf16_peak, "unit": "TFLOP/s", "frac": round(attn_tflops / bf16_peak, 4),
+                     "peak_kind": f"{peak_kind} bf16 burst", "traffic": None,
+                     "flops_per_launch": flops, "ms_per_launch": round(attn_ms, 4)},
+        "consolidate": {"bound": "hbm", "achieved": round(cons_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                        "frac": round(cons_gbs / hbm_peak, 4), "bytes_per_step": cons_bytes,
+                        "ms_per_step": round(cons_ms, 4), "plan_blocks": plan_blocks[-1]},
+        "region_ms": round(region0.elapsed_time(region1), 3),
+        "clocks": clocks,
+        "e2e": {"value": round(ws * LQ / (e2e_ms / 1e3), 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4)},
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_queries)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def cpu_baseline(n_queries: int = 48):
+    """The fp64 oracle as it stands, on this host's cores, on a bounded sample of the workload.
+
+    Sample: one full steady-state consolidation step (3 frames into a 21-entry
+    memory, all 12 heads, every token) plus attention for n_queries of the 4680
+    query rows over all 12 heads and 32,760 keys per head; the attention time is
+    scaled to the 4680 rows of one step.
+    """
+    from oracle import OracleMemory, oracle_num_threads
+    from synth import KIND_K, KIND_V, HostAR1, host_queries
+    elems = N * H * D
+    mem = OracleMemory(M, BETA, anchor=True, elems=elems)
+    gk = HostAR1((N, H, D), 7, KIND_K)
+    gv = HostAR1((N, H, D), 7, KIND_V)
+
+    def frame(g):
+        return torch.from_numpy(g.next()).to(torch.bfloat16).double().numpy()
+    for _ in range(M + 3):  # fill the budget and start merging
+        mem.insert(frame(gk), frame(gv))
+    new = [(frame(gk), frame(gv)) for _ in range(F)]
+    t0 = time.perf_counter()
+    for K, V in new:
+        mem.insert(K, V)
+    t_cons = time.perf_counter() - t0
+    Q = torch.from_numpy(host_queries((n_queries, H, D), 7)).to(torch.bfloat16).double().numpy()
+    t0 = time.perf_counter()
+    mem.attend(Q, N, H, D)
+    t_attn = time.perf_counter() - t0
+    step_s = t_cons + t_attn * (LQ / n_queries)
+    return {"value": round(LQ / step_s, 3), "unit": "tokens/s", "cores": oracle_num_threads(), "kind": "oracle",
+            "sample": f"fp64 C oracle: one full 3-frame consolidation (all heads/tokens) + attention of "
+                      f"{n_queries}/{LQ} query rows x {H} heads over {M * N} keys, scaled to {LQ} rows",
+            "seconds_measured": round(t_cons + t_attn, 2)}
+
+
+def run_reference(args):
+    """The oracle as the reference arm: each step a bounded sample of the same workload."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    times = []
+    base = None
+    for i in range(args.warmup + args.steps):
+        r = cpu_baseline(args.cpu_queries)
+        if i >= args.warmup:
+            times.append(LQ / r["value"])
+        base = r
+    step_s = statistics.mean(times)
+    value = LQ / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (AR(1) K/V rho=0.9, N(0,1) Q)",
+            "config": {"workload": WORKLOAD},
+            "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": base["cores"], "kind": "oracle",
+                             "sample": base["sample"]},
+            "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-queries", type=int, default=48)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_cuda(args)
+
+
+if __name__ == "__main__":
+    main()

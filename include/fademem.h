@@ -1,0 +1,175 @@
+/*
+ * fademem.h -- C ABI of the GB300 (sm_103a) implementation of FadeMem's
+ * per-segment memory step (arxiv 2606.10671, "FadeMem: Distance-Aware Memory
+ * Consolidation for Autoregressive Video Diffusion").
+ *
+ * The memory (Sec. 3.1) is an ordered set of at most M entries per layer.
+ * Each entry stores one representative K/V block of N tokens x H heads x D
+ * dims, its temporal centre mu and its span s (Sec. 3.3, "Memory entries").
+ * Each generated unit (one latent frame, Sec. S4) is inserted as a new entry;
+ * when the budget is exceeded, the power-law schedule picks the adjacent pair
+ * with the smallest warped gap |(t-mu_{i+1})^beta - (t-mu_i)^beta| and the
+ * pair is consolidated (Sec. 3.3; Algorithm S1).  The segment's queries then
+ * attend over the consolidated memory, per head and per layer (Sec. 3.3, last
+ * paragraph; Sec. 4.1: attention every denoising step, memory update after
+ * the last one).
+ *
+ * Conventions (every entry point):
+ *   - Returns a fademem_status; never aborts, never throws across the ABI.
+ *     On failure fademem_last_error() describes the problem (thread-local).
+ *   - Device pointers are CUDA device addresses; they must be 16-byte
+ *     aligned, else FADEMEM_ERR_INVALID_ARG.  Host pointers are plain memory.
+ *   - Work is enqueued asynchronously on the given stream (a cudaStream_t
+ *     passed as void*; NULL = the legacy default stream).  Calls that return
+ *     data to the host synchronise that stream first.
+ *   - A handle is not thread-safe; use one handle per thread or serialise.
+ *   - Frames are counted from t = 0 (the first inserted frame is the anchor).
+ */
+#ifndef FADEMEM_H
+#define FADEMEM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define FADEMEM_API __attribute__((visibility("default")))
+#else
+#define FADEMEM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Largest entry budget M accepted by fademem_create. */
+#define FADEMEM_MAX_BUDGET 64
+/* Largest number of layers one handle holds. */
+#define FADEMEM_MAX_LAYERS 128
+/* Largest number of frames pending (inserted, not yet consolidated) per layer. */
+#define FADEMEM_MAX_PENDING 64
+
+typedef enum fademem_status {
+    FADEMEM_OK = 0,
+    FADEMEM_ERR_INVALID_ARG = 1,    /* NULL / misaligned pointer, out-of-range size or index */
+    FADEMEM_ERR_UNSUPPORTED = 2,    /* valid but not implemented (e.g. bf16 with head_dim 64) */
+    FADEMEM_ERR_WORKSPACE = 3,      /* workspace too small or misaligned */
+    FADEMEM_ERR_EMPTY = 4,          /* attend on a memory with no entries */
+    FADEMEM_ERR_PENDING = 5,        /* attend while inserted frames await consolidation */
+    FADEMEM_ERR_CUDA = 6,           /* a CUDA runtime call failed (message has the CUDA error) */
+    FADEMEM_ERR_DEVICE_TIMEOUT = 7, /* a device-side bounded wait gave up (see device status) */
+    FADEMEM_ERR_DEVICE_CHECK = 8    /* a device-side consistency check failed */
+} fademem_status;
+
+typedef enum fademem_dtype {
+    FADEMEM_F32 = 0,   /* fp32 storage and arithmetic (exact reference path) */
+    FADEMEM_BF16 = 1   /* bf16 storage, fp32 accumulation; tensor-core attention */
+} fademem_dtype;
+
+/* Consolidation operator (Sec. 3.3; ablation of Table 2). */
+typedef enum fademem_merge_op {
+    FADEMEM_MERGE_WEIGHTED = 0,       /* default: weights sqrt(s_j), sqrt(s_{j+1}), normalised */
+    FADEMEM_MERGE_AVERAGE = 1,        /* unweighted mean of the two blocks */
+    FADEMEM_MERGE_SELECT_NEAREST = 2, /* keep the block of the entry nearer the current step (m_{j+1}) */
+    FADEMEM_MERGE_MAX_POOL = 3        /* elementwise maximum */
+} fademem_merge_op;
+
+typedef struct fademem_config {
+    int budget;            /* M: entries per layer, 2 <= M <= FADEMEM_MAX_BUDGET (Sec. 3.1) */
+    int heads;             /* H >= 1 */
+    int head_dim;          /* D: 64 or 128 (bf16 attention: 128) */
+    int tokens_per_frame;  /* N >= 1: tokens in one unit's KV block (Sec. 3.1) */
+    int num_layers;        /* L: 1 <= L <= FADEMEM_MAX_LAYERS; all layers share one schedule */
+    double beta;           /* warp exponent of u(d) = d^beta, 0 < beta <= 1 (Sec. 3.3) */
+    int anchor;            /* 1: keep the first frame as global anchor (Sec. 3.3; Algorithm S1) */
+    int merge_op;          /* fademem_merge_op */
+    int dtype;             /* fademem_dtype of K, V, Q, out and the stored memory */
+    float scale;           /* softmax scale of q.k; 0 selects 1/sqrt(D) */
+} fademem_config;
+
+typedef struct fademem_ctx *fademem_t;
+
+/* Bytes of device workspace a handle with this configuration needs (the
+ * memory of every layer, [L][K|V][H][M][N][D] in the storage dtype, plus
+ * metadata and the merge plan), or 0 if the configuration is invalid.
+ * Host only; no CUDA call. */
+FADEMEM_API size_t fademem_workspace_bytes(const fademem_config *cfg);
+
+/* Create a memory (Sec. 3.1: empty, |M_0| = 0) over caller-owned device
+ * workspace (>= fademem_workspace_bytes, 256-byte aligned).  The caller keeps
+ * ownership of the workspace and must keep it alive until fademem_destroy.
+ * Host only: the metadata is initialised by the first device call.
+ * Errors: INVALID_ARG (bad config, NULL out), UNSUPPORTED, WORKSPACE. */
+FADEMEM_API fademem_status fademem_create(const fademem_config *cfg, void *workspace, size_t workspace_bytes,
+                                          fademem_t *out);
+
+/* Register nframes new units for one layer (Sec. 3.3, "insertion": each unit
+ * becomes an entry (K_t, V_t, mu = t, s = 1)).  K and V are device arrays of
+ * [nframes * N][H][D] in the config dtype (token-major, frames in generation
+ * order).  No data moves here: the arrays are borrowed and must stay valid
+ * and unmodified until fademem_consolidate has been enqueued and the stream
+ * has reached it.  Every layer must register the same frames before the next
+ * consolidate.  Errors: INVALID_ARG, PENDING (over FADEMEM_MAX_PENDING). */
+FADEMEM_API fademem_status fademem_insert(fademem_t h, int layer, const void *K, const void *V, int nframes);
+
+/* Apply Algorithm S1 once per pending frame, in order, to every layer:
+ * append, and while over budget compute the warped gaps on the device, take
+ * the argmin (lowest index on ties) over the eligible pairs (all but the pair
+ * holding the newest entry), merge its span/centre (anchor rule for the pair
+ * holding the first frame), and consolidate the pair's K/V blocks in place.
+ * Consecutive frames are fused into one pass over the memory (each source
+ * block read once, each changed slot written once).  Asynchronous on stream.
+ * Storage slots: the merged entry keeps m_j's slot, the new entry takes
+ * m_{j+1}'s; occupied slots are always 0..count-1.
+ * Errors: INVALID_ARG (layers with different pending frames), CUDA. */
+FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void *stream);
+
+/* Attention of Lq query tokens over every token of every entry of one layer,
+ * per head: out = softmax(scale * Q K^T) V (keys and values of all count*N
+ * cached tokens; non-causal, all cached keys precede the queries).  Q, out:
+ * device arrays [Lq][H][D] in the config dtype.  Asynchronous on stream.
+ * Errors: INVALID_ARG, EMPTY (no entries), PENDING (frames not consolidated),
+ * UNSUPPORTED, CUDA. */
+FADEMEM_API fademem_status fademem_attend(fademem_t h, int layer, const void *Q, void *out, int Lq, void *stream);
+
+/* Number of entries (count = min(frames seen, M)) and frames seen so far,
+ * counting consolidated frames only.  Host only. */
+FADEMEM_API fademem_status fademem_counts(fademem_t h, int *count, int64_t *frames_seen);
+
+/* Copy the entry table back, in temporal order (synchronises stream):
+ * slot (storage slot of entry i), first (first unit summarised), span (s),
+ * mu2 (2*mu, exact integer).  Arrays hold >= capacity elements; *count gets
+ * the number of entries.  Errors: INVALID_ARG (capacity too small), CUDA. */
+FADEMEM_API fademem_status fademem_get_entries(fademem_t h, void *stream, int capacity, int *count, int32_t *slot,
+                                               int64_t *first, int64_t *span, int64_t *mu2);
+
+/* Size of the most recent consolidation pass's merge plan (synchronises
+ * stream): *n_src source blocks read (old entries and new frames), *n_dest
+ * slots written, *frames units in the pass.  Each block is N*H*D elements of
+ * K plus as many of V per layer, so the pass moves (n_src + n_dest) blocks of
+ * K and V per layer: the algorithmic HBM traffic of the consolidation. */
+FADEMEM_API fademem_status fademem_last_plan(fademem_t h, void *stream, int *n_src, int *n_dest, int *frames);
+
+/* Device pointers to one layer's stored K and V memory, each laid out as
+ * [H][M][N][D] in the storage dtype; storage slot s of head h starts at
+ * ((h * M) + s) * N * D elements.  Only slots 0..count-1 hold entries. */
+FADEMEM_API fademem_status fademem_layer_memory(fademem_t h, int layer, void **K, void **V);
+
+/* Read and clear the device status word (synchronises stream).  Returns OK,
+ * DEVICE_TIMEOUT (a bounded wait in a kernel gave up) or DEVICE_CHECK; the
+ * raw word goes to *word when word is not NULL. */
+FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void *stream, uint32_t *word);
+
+/* Forget every entry (count = 0, t = 0).  Enqueued on stream. */
+FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
+
+/* Release the handle (NULL-safe).  Does not free the caller's workspace. */
+FADEMEM_API void fademem_destroy(fademem_t h);
+
+/* Message of the last failed call on this thread ("" if none). */
+FADEMEM_API const char *fademem_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FADEMEM_H */

@@ -1,0 +1,69 @@
+// fp32 attention of query tokens over the memory (Sec. 3.3 last paragraph:
+// the memory is the cached context the backbone's attention sees).
+// Exact-precision path for the fp32 storage dtype: one warp per (query, head),
+// lanes split the head dimension, online softmax over every cached key in
+// fp32 (tf32 tensor cores would not meet a 1e-5 relative tolerance).
+#include <math.h>
+
+#include "fademem_internal.h"
+
+namespace fademem {
+namespace {
+
+template <int D>
+__global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict__ Kc, const float* __restrict__ Vc,
+                                                         const float* __restrict__ Q, float* __restrict__ out,
+                                                         int Lq, int Lk, int H, size_t head_stride,
+                                                         float scale_log2) {
+  constexpr int P = D / 32;
+  const int lane = threadIdx.x & 31;
+  const long long gw = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  if (gw >= (long long)Lq * H) return;
+  const int q = (int)(gw / H), h = (int)(gw % H);
+  const float* qp = Q + ((size_t)q * H + h) * D;
+  float qv[P], o[P];
+#pragma unroll
+  for (int i = 0; i < P; ++i) { qv[i] = qp[lane + 32 * i]; o[i] = 0.f; }
+  const float* Kh = Kc + (size_t)h * head_stride;  // keys of head h: [Lk][D], slots 0..count-1 contiguous
+  const float* Vh = Vc + (size_t)h * head_stride;
+  float m = -INFINITY, l = 0.f;
+  for (int k = 0; k < Lk; ++k) {
+    float dot = 0.f;
+#pragma unroll
+    for (int i = 0; i < P; ++i) dot = fmaf(qv[i], Kh[(size_t)k * D + lane + 32 * i], dot);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    const float s = dot * scale_log2;
+    const float m_new = fmaxf(m, s);
+    const float c = exp2f(m - m_new);
+    const float p = exp2f(s - m_new);
+    l = l * c + p;
+#pragma unroll
+    for (int i = 0; i < P; ++i) o[i] = fmaf(p, Vh[(size_t)k * D + lane + 32 * i], o[i] * c);
+    m = m_new;
+  }
+  float* op = out + ((size_t)q * H + h) * D;
+  const float inv = 1.f / l;
+#pragma unroll
+  for (int i = 0; i < P; ++i) op[lane + 32 * i] = o[i] * inv;
+}
+
+}  // namespace
+
+cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, const float* Q, float* out,
+                              int Lq, int Lk, float scale, cudaStream_t stream) {
+  const long long warps = (long long)Lq * g.H;
+  const int threads = 256;
+  const long long blocks = (warps * 32 + threads - 1) / threads;
+  const float scale_log2 = scale * 1.4426950408889634f;
+  const size_t head_stride = (size_t)g.M * g.N * g.D;
+  if (g.D == 128)
+    attend_f32_kernel<128><<<(unsigned)blocks, threads, 0, stream>>>(
+        (const float*)Kc, (const float*)Vc, Q, out, Lq, Lk, g.H, head_stride, scale_log2);
+  else
+    attend_f32_kernel<64><<<(unsigned)blocks, threads, 0, stream>>>(
+        (const float*)Kc, (const float*)Vc, Q, out, Lq, Lk, g.H, head_stride, scale_log2);
+  return cudaGetLastError();
+}
+
+}  // namespace fademem

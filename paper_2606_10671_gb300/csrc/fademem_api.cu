@@ -1,0 +1,331 @@
+// C ABI of the FadeMem library (include/fademem.h): argument checks, workspace
+// layout, the pending-insert list and the split of pending frames into fused
+// passes.  All arithmetic of the method runs in the kernels.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <new>
+#include <vector>
+
+#include "fademem_internal.h"
+
+using namespace fademem;
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+fademem_status fail(fademem_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+fademem_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(FADEMEM_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Chunk {
+  const char* K;
+  const char* V;
+  int frames;
+};
+
+}  // namespace
+
+struct fademem_ctx {
+  fademem_config cfg;
+  Geometry g;
+  char* ws;
+  size_t ws_bytes;
+  DevState* st;
+  char* cache;
+  bool need_init;
+  int count;             // entries, = min(frames, M) (one merge per insert beyond the budget)
+  long long frames;      // consolidated frames
+  std::vector<Chunk> pending[FADEMEM_MAX_LAYERS];
+  int pending_frames[FADEMEM_MAX_LAYERS];
+};
+
+static fademem_status check_config(const fademem_config* c, Geometry* g) {
+  if (!c) return fail(FADEMEM_ERR_INVALID_ARG, "config is NULL");
+  if (c->budget < 2 || c->budget > FADEMEM_MAX_BUDGET)
+    return fail(FADEMEM_ERR_INVALID_ARG, "budget must be in [2, %d] (got %d)", FADEMEM_MAX_BUDGET, c->budget);
+  if (c->heads < 1 || c->heads > 65535) return fail(FADEMEM_ERR_INVALID_ARG, "heads must be >= 1 (got %d)", c->heads);
+  if (c->head_dim != 64 && c->head_dim != 128)
+    return fail(FADEMEM_ERR_INVALID_ARG, "head_dim must be 64 or 128 (got %d)", c->head_dim);
+  if (c->tokens_per_frame < 1 || c->tokens_per_frame > (1 << 20))
+    return fail(FADEMEM_ERR_INVALID_ARG, "tokens_per_frame must be in [1, 2^20] (got %d)", c->tokens_per_frame);
+  if (c->num_layers < 1 || c->num_layers > FADEMEM_MAX_LAYERS)
+    return fail(FADEMEM_ERR_INVALID_ARG, "num_layers must be in [1, %d] (got %d)", FADEMEM_MAX_LAYERS,
+                c->num_layers);
+  if (!(c->beta > 0.0 && c->beta <= 1.0)) return fail(FADEMEM_ERR_INVALID_ARG, "beta must be in (0, 1]");
+  if (c->anchor != 0 && c->anchor != 1) return fail(FADEMEM_ERR_INVALID_ARG, "anchor must be 0 or 1");
+  if (c->merge_op < 0 || c->merge_op > 3) return fail(FADEMEM_ERR_INVALID_ARG, "unknown merge_op %d", c->merge_op);
+  if (c->dtype != FADEMEM_F32 && c->dtype != FADEMEM_BF16)
+    return fail(FADEMEM_ERR_INVALID_ARG, "unknown dtype %d", c->dtype);
+  if (!(c->scale >= 0.f) || isinf(c->scale)) return fail(FADEMEM_ERR_INVALID_ARG, "scale must be finite and >= 0");
+  if (c->dtype == FADEMEM_BF16 && c->head_dim != 128)
+    return fail(FADEMEM_ERR_UNSUPPORTED, "bf16 storage supports head_dim 128 only");
+  const long long lk = (long long)c->budget * c->tokens_per_frame;
+  if (lk > (1LL << 30)) return fail(FADEMEM_ERR_INVALID_ARG, "budget * tokens_per_frame too large");
+  if (g) {
+    g->L = c->num_layers;
+    g->H = c->heads;
+    g->M = c->budget;
+    g->N = c->tokens_per_frame;
+    g->D = c->head_dim;
+    g->dtype = c->dtype;
+    g->elem = c->dtype == FADEMEM_BF16 ? 2 : 4;
+    g->slab_elems = (size_t)g->N * g->D;
+    g->kv_elems = (size_t)g->H * g->M * g->slab_elems;
+    g->state_bytes = round_up(sizeof(DevState), 256);
+    g->layer_bytes = round_up(2 * g->kv_elems * g->elem, 256);
+    g->total_bytes = g->state_bytes + (size_t)g->L * g->layer_bytes;
+  }
+  return FADEMEM_OK;
+}
+
+extern "C" {
+
+FADEMEM_API size_t fademem_workspace_bytes(const fademem_config* cfg) {
+  Geometry g;
+  if (check_config(cfg, &g) != FADEMEM_OK) return 0;
+  return g.total_bytes;
+}
+
+FADEMEM_API fademem_status fademem_create(const fademem_config* cfg, void* workspace, size_t workspace_bytes,
+                                          fademem_t* out) {
+  if (!out) return fail(FADEMEM_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  Geometry g;
+  fademem_status s = check_config(cfg, &g);
+  if (s != FADEMEM_OK) return s;
+  if (!workspace) return fail(FADEMEM_ERR_WORKSPACE, "workspace is NULL");
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+    return fail(FADEMEM_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  if (workspace_bytes < g.total_bytes)
+    return fail(FADEMEM_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, g.total_bytes);
+  fademem_ctx* h = new (std::nothrow) fademem_ctx();
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "out of host memory");
+  h->cfg = *cfg;
+  if (h->cfg.scale == 0.f) h->cfg.scale = 1.0f / sqrtf((float)cfg->head_dim);
+  h->g = g;
+  h->ws = reinterpret_cast<char*>(workspace);
+  h->ws_bytes = workspace_bytes;
+  h->st = reinterpret_cast<DevState*>(h->ws);
+  h->cache = h->ws + g.state_bytes;
+  h->need_init = true;
+  h->count = 0;
+  h->frames = 0;
+  for (int l = 0; l < FADEMEM_MAX_LAYERS; ++l) h->pending_frames[l] = 0;
+  *out = h;
+  g_err[0] = 0;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_insert(fademem_t h, int layer, const void* K, const void* V, int nframes) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (!K || !V) return fail(FADEMEM_ERR_INVALID_ARG, "K or V is NULL");
+  if (!aligned16(K) || !aligned16(V)) return fail(FADEMEM_ERR_INVALID_ARG, "K and V must be 16-byte aligned");
+  if (nframes < 1) return fail(FADEMEM_ERR_INVALID_ARG, "nframes must be >= 1 (got %d)", nframes);
+  if (h->pending_frames[layer] + nframes > FADEMEM_MAX_PENDING)
+    return fail(FADEMEM_ERR_PENDING, "more than %d frames pending on layer %d", FADEMEM_MAX_PENDING, layer);
+  h->pending[layer].push_back(Chunk{reinterpret_cast<const char*>(K), reinterpret_cast<const char*>(V), nframes});
+  h->pending_frames[layer] += nframes;
+  return FADEMEM_OK;
+}
+
+static fademem_status ensure_init(fademem_t h, cudaStream_t stream) {
+  if (!h->need_init) return FADEMEM_OK;
+  cudaError_t e = cudaMemsetAsync(h->st, 0, sizeof(DevState), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "initialising the entry table");
+  h->need_init = false;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  const int L = h->g.L;
+  const int F = h->pending_frames[0];
+  for (int l = 1; l < L; ++l)
+    if (h->pending_frames[l] != F)
+      return fail(FADEMEM_ERR_INVALID_ARG, "layer %d has %d pending frames, layer 0 has %d", l,
+                  h->pending_frames[l], F);
+  if (F == 0) return FADEMEM_OK;
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+
+  const size_t frame_bytes = (size_t)h->g.N * h->g.H * h->g.D * h->g.elem;
+  std::vector<int> ci(L, 0), co(L, 0);  // chunk index and frame offset inside it, per layer
+  PassSources srcs;
+  memset(&srcs, 0, sizeof(srcs));
+  int done = 0;
+  while (done < F) {
+    int nf = F - done < kMaxPassFrames ? F - done : kMaxPassFrames;
+    for (int l = 0; l < L; ++l) {
+      const int left = h->pending[l][ci[l]].frames - co[l];
+      if (left < nf) nf = left;  // a pass never crosses an insert boundary
+    }
+    for (int l = 0; l < L; ++l) {
+      const Chunk& c = h->pending[l][ci[l]];
+      srcs.src[l][0] = c.K + (size_t)co[l] * frame_bytes;
+      srcs.src[l][1] = c.V + (size_t)co[l] * frame_bytes;
+    }
+    cudaError_t e = launch_schedule(h->st, nf, h->g.M, h->cfg.beta, h->cfg.anchor, h->cfg.merge_op, h->count,
+                                    stream);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the schedule kernel");
+    e = launch_consolidate(h->g, h->cache, h->st, srcs, nf, h->cfg.merge_op, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the consolidation kernel");
+    h->frames += nf;
+    h->count = h->frames < h->g.M ? (int)h->frames : h->g.M;
+    for (int l = 0; l < L; ++l) {
+      co[l] += nf;
+      if (co[l] == h->pending[l][ci[l]].frames) {
+        ++ci[l];
+        co[l] = 0;
+      }
+    }
+    done += nf;
+  }
+  for (int l = 0; l < L; ++l) {
+    h->pending[l].clear();
+    h->pending_frames[l] = 0;
+  }
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_attend(fademem_t h, int layer, const void* Q, void* out, int Lq, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
+  if (!Q || !out) return fail(FADEMEM_ERR_INVALID_ARG, "Q or out is NULL");
+  if (!aligned16(Q) || !aligned16(out)) return fail(FADEMEM_ERR_INVALID_ARG, "Q and out must be 16-byte aligned");
+  if (Lq < 1 || Lq > (1 << 24)) return fail(FADEMEM_ERR_INVALID_ARG, "Lq must be in [1, 2^24] (got %d)", Lq);
+  for (int l = 0; l < h->g.L; ++l)
+    if (h->pending_frames[l] != 0)
+      return fail(FADEMEM_ERR_PENDING, "frames inserted on layer %d await fademem_consolidate", l);
+  if (h->count == 0) return fail(FADEMEM_ERR_EMPTY, "the memory holds no entries");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  const int Lk = h->count * h->g.N;
+  const char* Kc = h->cache + (size_t)layer * h->g.layer_bytes;
+  const char* Vc = Kc + h->g.kv_elems * h->g.elem;
+  cudaError_t e;
+  if (h->g.dtype == FADEMEM_F32) {
+    e = launch_attend_f32(h->g, Kc, Vc, reinterpret_cast<const float*>(Q), reinterpret_cast<float*>(out), Lq, Lk,
+                          h->cfg.scale, stream);
+  } else {
+    char msg[256] = "";
+    e = launch_attend_bf16(h->g, Kc, Vc, Q, out, Lq, Lk, h->cfg.scale, &h->st->status, stream, msg, sizeof(msg));
+    if (e == cudaErrorNotSupported) return fail(FADEMEM_ERR_UNSUPPORTED, "%s", msg);
+    if (e == cudaErrorInvalidValue && msg[0]) return fail(FADEMEM_ERR_INVALID_ARG, "%s", msg);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "launching the attention kernel");
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_counts(fademem_t h, int* count, int64_t* frames_seen) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (count) *count = h->count;
+  if (frames_seen) *frames_seen = h->frames;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_get_entries(fademem_t h, void* stream_, int capacity, int* count, int32_t* slot,
+                                               int64_t* first, int64_t* span, int64_t* mu2) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (!count) return fail(FADEMEM_ERR_INVALID_ARG, "count is NULL");
+  if (capacity < h->count) return fail(FADEMEM_ERR_INVALID_ARG, "capacity %d < %d entries", capacity, h->count);
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  DevMeta m;
+  e = cudaMemcpy(&m, &h->st->meta, sizeof(m), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the entry table");
+  if (m.count < 0 || m.count > kMaxEntries)
+    return fail(FADEMEM_ERR_DEVICE_CHECK, "device entry count %d is out of range", m.count);
+  if (m.count > capacity) return fail(FADEMEM_ERR_INVALID_ARG, "capacity %d < %d entries", capacity, m.count);
+  *count = m.count;
+  for (int i = 0; i < m.count; ++i) {
+    if (slot) slot[i] = m.slot[i];
+    if (first) first[i] = m.first[i];
+    if (span) span[i] = m.span[i];
+    if (mu2) mu2[i] = (int64_t)llround(2.0 * m.mu[i]);
+  }
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_last_plan(fademem_t h, void* stream_, int* n_src, int* n_dest, int* frames) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  DevPlan p;
+  e = cudaMemcpy(&p, &h->st->plan, sizeof(p), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the merge plan");
+  if (n_src) *n_src = p.n_src;
+  if (n_dest) *n_dest = p.n_dest;
+  if (frames) *frames = p.frames;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_layer_memory(fademem_t h, int layer, void** K, void** V) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
+  char* k = h->cache + (size_t)layer * h->g.layer_bytes;
+  if (K) *K = k;
+  if (V) *V = k + h->g.kv_elems * h->g.elem;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void* stream_, uint32_t* word) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  unsigned int w = 0;
+  e = cudaMemcpy(&w, &h->st->status, sizeof(w), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the device status");
+  const unsigned int zero = 0;
+  e = cudaMemcpy(&h->st->status, &zero, sizeof(zero), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
+  if (word) *word = w;
+  if (w & kStatusTimeout) return fail(FADEMEM_ERR_DEVICE_TIMEOUT, "a device wait timed out (status 0x%x)", w);
+  if (w) return fail(FADEMEM_ERR_DEVICE_CHECK, "a device check failed (status 0x%x)", w);
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->need_init = true;
+  fademem_status s = ensure_init(h, reinterpret_cast<cudaStream_t>(stream_));
+  if (s != FADEMEM_OK) return s;
+  h->count = 0;
+  h->frames = 0;
+  for (int l = 0; l < h->g.L; ++l) {
+    h->pending[l].clear();
+    h->pending_frames[l] = 0;
+  }
+  return FADEMEM_OK;
+}
+
+FADEMEM_API void fademem_destroy(fademem_t h) { delete h; }
+
+FADEMEM_API const char* fademem_last_error(void) { return g_err; }
+
+}  // extern "C"

@@ -1,0 +1,90 @@
+// Internal declarations of the FadeMem CUDA library (not part of the C ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/fademem.h"
+
+namespace fademem {
+
+// Frames fused into one schedule + consolidation pass.  A pass of F frames
+// changes at most 2F slots (merged entry + new entry per frame) and reads at
+// most 3F sources (two old blocks per merge + one new frame each).
+constexpr int kMaxPassFrames = 4;
+constexpr int kMaxDest = 2 * kMaxPassFrames;
+constexpr int kMaxSrc = 3 * kMaxPassFrames;
+constexpr int kMaxEntries = FADEMEM_MAX_BUDGET + 1;
+
+// Device status word bits (fademem_get_device_status).
+constexpr uint32_t kStatusTimeout = 1u << 0;      // a bounded mbarrier wait gave up
+constexpr uint32_t kStatusCountMismatch = 1u << 1;  // host and device entry counts disagree
+constexpr uint32_t kStatusPlanOverflow = 1u << 2;  // merge plan exceeded its static bounds
+
+// Entry table of the memory (Sec. 3.3 "memory entries"), temporal order.
+struct DevMeta {
+  int count;
+  int pad0;
+  long long t_next;                  // index of the next unit (frames seen)
+  int slot[kMaxEntries];             // storage slot of entry i
+  long long first[kMaxEntries];      // first unit summarised
+  long long span[kMaxEntries];       // s
+  double mu[kMaxEntries];            // temporal centre
+};
+
+// Fused merge plan of one pass.  Destination d receives
+//   sum_k w_k * source_k   (linear operators)   or   max_k source_k (max pooling)
+// over its sources, which are stored contiguously and in destination order.
+// A source is an old slot (ref >= 0, its content before the pass) or a new
+// frame of the pass (ref = -(f + 1)).
+struct DevPlan {
+  int n_src;
+  int n_dest;
+  int frames;
+  int op;
+  int src_ref[kMaxSrc];
+  float src_w[kMaxSrc];
+  int src_dest[kMaxSrc];
+  int dest_slot[kMaxDest];
+  int merged_pair[kMaxPassFrames];   // j chosen for each frame (-1: no merge)
+};
+
+struct DevState {
+  DevMeta meta;
+  DevPlan plan;
+  unsigned int status;
+  unsigned int pad[7];
+};
+
+// Layout of one layer in the workspace: K then V, each [H][M][N][D].
+struct Geometry {
+  int L, H, M, N, D;
+  int dtype;             // fademem_dtype
+  size_t elem;           // bytes per element
+  size_t slab_elems;     // N * D
+  size_t kv_elems;       // H * M * N * D (one of K or V of one layer)
+  size_t state_bytes;    // DevState, rounded to 256
+  size_t layer_bytes;    // 2 * kv_elems * elem, rounded to 256
+  size_t total_bytes;
+};
+
+// Per-pass source pointers: layer l's K (or V) frames of the pass start at
+// src[l][0] (K) / src[l][1] (V), frames contiguous ([F*N][H][D]).
+struct PassSources {
+  const void* src[FADEMEM_MAX_LAYERS][2];
+};
+
+// expected_count: the host's entry count before the pass (count = min(frames, M));
+// a mismatch sets kStatusCountMismatch in the device status word.
+cudaError_t launch_schedule(DevState* st, int frames, int M, double beta, int anchor, int op, int expected_count,
+                            cudaStream_t stream);
+cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
+                               int frames, int op, cudaStream_t stream);
+cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, const float* Q, float* out,
+                              int Lq, int Lk, float scale, cudaStream_t stream);
+// Returns cudaErrorNotSupported if the shape is outside the tensor-core path.
+cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, const void* Q, void* out, int Lq,
+                               int Lk, float scale, unsigned int* status, cudaStream_t stream,
+                               char* err, size_t errlen);
+
+}  // namespace fademem

@@ -1,0 +1,126 @@
+"""Drive the CUDA memory (through the C ABI) and the fp64 oracle side by side.
+
+Both sides consume exactly the same inputs: frames drawn by synth/, rounded to
+the storage dtype, uploaded for the device and widened to fp64 for the oracle.
+No oracle input or expected value is ever taken from the CUDA path.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import OracleMemory
+from synth import KIND_K, KIND_V, DeviceAR1, HostAR1, host_queries, rho_const
+
+OPS = {"weighted": 0, "average": 1, "select_nearest": 2, "max_pool": 3}
+
+# Tolerances (checked as written here):
+#   fp32 outputs and memory: max|gpu - oracle| <= 1e-5 * max|oracle|
+#   bf16 outputs and memory: max|gpu - oracle| <= 2e-2 (unit-variance data)
+F32_RTOL = 1e-5
+BF16_ATOL = 2e-2
+
+
+def assert_close(got: np.ndarray, ref: np.ndarray, dtype, what=""):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert got.shape == ref.shape, (what, got.shape, ref.shape)
+    assert np.all(np.isfinite(got)), what
+    err = np.max(np.abs(got - ref)) if got.size else 0.0
+    if dtype == torch.float32:
+        bound = F32_RTOL * max(np.max(np.abs(ref)), 1e-30)
+    else:
+        bound = BF16_ATOL
+    assert err <= bound, f"{what}: max|diff| {err:.3e} > {bound:.3e}"
+    return err
+
+
+class Pair:
+    """One FadeMem memory on the GPU and one oracle per layer, fed identical frames."""
+
+    def __init__(self, budget, heads, head_dim, tokens, beta=0.3, anchor=True, op="weighted",
+                 dtype=torch.bfloat16, layers=1, seed=0, rho=rho_const(0.9), tracked_heads=None, device_gen=False):
+        from paper_2606_10671_gb300 import FadeMem
+        self.M, self.H, self.D, self.N, self.L = budget, heads, head_dim, tokens, layers
+        self.dtype = dtype
+        self.tracked = list(range(heads)) if tracked_heads is None else list(tracked_heads)
+        self.gpu = FadeMem(budget, heads, head_dim, tokens, num_layers=layers, beta=beta, anchor=anchor, merge_op=op,
+                           dtype=dtype)
+        elems = tokens * len(self.tracked) * head_dim
+        self.ora = [OracleMemory(budget, beta, anchor=anchor, op=OPS[op], elems=elems) for _ in range(layers)]
+        shape = (tokens, heads, head_dim)
+        if device_gen:
+            self.gens = [(DeviceAR1(shape, seed, KIND_K, l, rho, dtype), DeviceAR1(shape, seed, KIND_V, l, rho, dtype))
+                         for l in range(layers)]
+        else:
+            self.gens = [(HostAR1(shape, seed, KIND_K, l, rho), HostAR1(shape, seed, KIND_V, l, rho))
+                         for l in range(layers)]
+        self.device_gen = device_gen
+        self.seed = seed
+
+    def _frames(self, gen, n):
+        if self.device_gen:
+            return torch.stack([gen.next() for _ in range(n)]).contiguous()
+        x = np.stack([gen.next() for _ in range(n)])
+        return torch.from_numpy(x).to(self.dtype).cuda()
+
+    def insert(self, frames: int, per_call: int | None = None):
+        """Insert `frames` frames on every layer (in calls of `per_call` frames), without consolidating."""
+        per_call = per_call or frames
+        for l in range(self.L):
+            gk, gv = self.gens[l]
+            K = self._frames(gk, frames)
+            V = self._frames(gv, frames)
+            for a in range(0, frames, per_call):
+                b = min(frames, a + per_call)
+                self.gpu.insert(l, K[a:b].contiguous(), V[a:b].contiguous())
+            Kt = K[:, :, self.tracked, :].double().cpu().numpy()
+            Vt = V[:, :, self.tracked, :].double().cpu().numpy()
+            for f in range(frames):
+                self.ora[l].insert(Kt[f], Vt[f])
+            self._keep = (K, V)
+
+    def step(self, frames: int = 3, per_call: int | None = None):
+        self.insert(frames, per_call)
+        self.gpu.consolidate()
+
+    def check_entries(self):
+        slot, first, span, mu2 = self.gpu.entries()
+        o_slot, o_first, o_span, o_mu = self.ora[0].entries()
+        assert slot.tolist() == o_slot.tolist(), (slot, o_slot)
+        assert first.tolist() == o_first.tolist()
+        assert span.tolist() == o_span.tolist()
+        assert mu2.tolist() == [int(round(2 * m)) for m in o_mu]
+        assert np.all(2 * o_mu == np.round(2 * o_mu))
+        return slot
+
+    def check_memory(self, layer=0):
+        """Every stored block of every entry, for the tracked heads."""
+        Kd, Vd = self.gpu.layer_memory(layer)
+        ora = self.ora[layer]
+        slot, _, _, _ = ora.entries()
+        worst = 0.0
+        for i, s in enumerate(slot.tolist()):
+            Ko, Vo = ora.entry_kv(i)
+            Ko = Ko.reshape(self.N, len(self.tracked), self.D).transpose(1, 0, 2)
+            Vo = Vo.reshape(self.N, len(self.tracked), self.D).transpose(1, 0, 2)
+            kg = Kd[self.tracked, s].double().cpu().numpy()
+            vg = Vd[self.tracked, s].double().cpu().numpy()
+            worst = max(worst, assert_close(kg, Ko, self.dtype, f"K entry {i} slot {s}"),
+                        assert_close(vg, Vo, self.dtype, f"V entry {i} slot {s}"))
+        return worst
+
+    def queries(self, Lq, step=0, layer=0):
+        q = host_queries((Lq, self.H, self.D), self.seed, layer, step)
+        return torch.from_numpy(q).to(self.dtype).cuda()
+
+    def check_attend(self, Q: torch.Tensor, layer=0, rows=None):
+        out = self.gpu.attend(layer, Q)
+        torch.cuda.synchronize()
+        Qh = Q.double().cpu().numpy()
+        og = out.double().cpu().numpy()
+        if rows is not None:
+            Qh, og = Qh[rows], og[rows]
+        Qt = Qh[:, self.tracked, :]
+        ref = self.ora[layer].attend(Qt, self.N, len(self.tracked), self.D)
+        return assert_close(og[:, self.tracked, :], ref, self.dtype, "attention")

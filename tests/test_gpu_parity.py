@@ -1,0 +1,142 @@
+"""CUDA path vs the fp64 oracle, element by element, through the C ABI (GPU only).
+
+Bar: slot table, first frame, span and 2*mu bit-exact after every consolidate;
+fp32 memory and outputs within 1e-5 relative (max-norm); bf16 within 2e-2
+max-abs on unit-variance data.
+"""
+import numpy as np
+import pytest
+import torch
+
+from synth import rho_const, rho_drift
+
+from parity_utils import Pair, assert_close
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built(cuda_lib):
+    from paper_2606_10671_gb300 import capi
+    capi.load(cuda_lib)
+
+
+def test_tiny_fp32_full_parity():
+    """Tiny config: fp32, 1 layer, 2 heads, D=64, N=64, 3-frame segments, M=8, 12 segments, rho=0.9, seed 0."""
+    p = Pair(8, 2, 64, 64, beta=0.3, dtype=torch.float32, seed=0)
+    for seg in range(12):
+        p.step(3)
+        p.check_entries()
+        p.check_memory()
+        p.check_attend(p.queries(192, step=seg))
+    assert p.gpu.counts() == (8, 36)
+    st, word = p.gpu.device_status()
+    assert word == 0
+
+
+def test_bf16_ragged_tiles():
+    """bf16 tensor-core path: N=100 (keys 500 = 3 tiles + 116), Lq=300 (2 tiles + 44), 3 heads."""
+    p = Pair(5, 3, 128, 100, beta=0.3, dtype=torch.bfloat16, seed=1)
+    for seg in range(8):
+        p.step(3)
+        p.check_entries()
+        p.check_memory()
+        p.check_attend(p.queries(300, step=seg))
+    p.gpu.device_status()
+
+
+@pytest.mark.parametrize("N,Lq,frames", [(50, 1, 1), (64, 128, 2), (1, 7, 1), (128, 256, 4), (37, 129, 3)])
+def test_bf16_attention_edges(N, Lq, frames):
+    """Fewer keys than one tile, exact tiles, one token per frame, a single query."""
+    p = Pair(4, 2, 128, N, beta=0.3, dtype=torch.bfloat16, seed=2)
+    p.step(frames)
+    p.check_entries()
+    p.check_attend(p.queries(Lq))
+    p.step(frames)
+    p.check_memory()
+    p.check_attend(p.queries(Lq, step=1))
+
+
+@pytest.mark.parametrize("op", ["weighted", "average", "select_nearest", "max_pool"])
+@pytest.mark.parametrize("anchor", [True, False])
+def test_merge_operators_fp32(op, anchor):
+    """The four consolidation operators of Table 2, with and without the first-frame anchor."""
+    p = Pair(5, 2, 64, 16, beta=0.3, anchor=anchor, op=op, dtype=torch.float32, seed=3)
+    for seg in range(10):
+        p.step(3)
+        p.check_entries()
+        p.check_memory()
+    p.check_attend(p.queries(40))
+
+
+@pytest.mark.parametrize("beta", [0.1, 0.5, 0.7, 0.9, 1.0])
+def test_beta_values(beta):
+    """Schedule exponents of the ablation (Table 2) and beta=1, whose gaps tie exactly."""
+    p = Pair(6, 1, 64, 8, beta=beta, dtype=torch.float32, seed=4)
+    for seg in range(40):
+        p.step(3)
+        p.check_entries()
+    p.check_memory()
+
+
+@pytest.mark.parametrize("per_call,frames", [(1, 3), (3, 3), (2, 7), (7, 7), (5, 13)])
+def test_insert_granularity(per_call, frames):
+    """Frames inserted in several calls and consolidated together (passes of <= 4 frames,
+    split at insert boundaries) give Algorithm S1's sequential result."""
+    p = Pair(4, 2, 64, 8, beta=0.3, dtype=torch.float32, seed=5)
+    for _ in range(6):
+        p.step(frames, per_call=per_call)
+        p.check_entries()
+        p.check_memory()
+
+
+def test_minimum_budget_and_multilayer():
+    """M=2 (one eligible pair), three layers with independent data sharing one schedule."""
+    p = Pair(2, 2, 64, 16, beta=0.3, dtype=torch.float32, layers=3, seed=6)
+    for seg in range(8):
+        p.step(3)
+        p.check_entries()
+        for l in range(3):
+            p.check_memory(l)
+    for l in range(3):
+        p.check_attend(p.queries(20, layer=l), layer=l)
+
+
+def test_status_codes_on_gpu():
+    from paper_2606_10671_gb300 import capi
+    p = Pair(4, 2, 128, 16, dtype=torch.bfloat16, seed=7)
+    Q = p.queries(16)
+    with pytest.raises(capi.FadeMemError) as e:
+        p.gpu.attend(0, Q)
+    assert e.value.status == capi.FADEMEM_ERR_EMPTY
+    p.insert(3)
+    with pytest.raises(capi.FadeMemError) as e:
+        p.gpu.attend(0, Q)
+    assert e.value.status == capi.FADEMEM_ERR_PENDING
+    p.gpu.consolidate()
+    p.check_attend(Q)
+    p.gpu.reset()
+    assert p.gpu.counts() == (0, 0)
+    slot, first, span, mu2 = p.gpu.entries()
+    assert len(slot) == 0
+
+
+def test_wan13b_single_layer_full_size():
+    """Wan-1.3B shape (H=12, D=128, N=1560, M=21, Lq=4680), the launch the bench times.
+
+    40 warm-up segments bring the memory to steady state (3 merges per segment);
+    the oracle tracks heads 0 and 11 in full, so every stored block of those heads
+    and 64 sampled query rows of the attention are compared exactly element by element.
+    """
+    p = Pair(21, 12, 128, 1560, beta=0.3, dtype=torch.bfloat16, seed=0, tracked_heads=[0, 11], device_gen=True)
+    for seg in range(40):
+        p.step(3)
+    p.check_entries()
+    p.check_memory()
+    rng = np.random.default_rng(0)
+    rows = np.sort(rng.choice(4680, 64, replace=False))
+    rows = np.unique(np.concatenate([rows, [0, 4679]]))
+    Q = p.queries(4680, step=40)
+    p.check_attend(Q, rows=rows)
+    p.gpu.device_status()
