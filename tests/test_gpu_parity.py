@@ -122,6 +122,18 @@ def test_status_codes_on_gpu():
     assert len(slot) == 0
 
 
+def test_wan13b_shape_fp32_storage_full_size():
+    """Wan-1.3B shape with fp32 storage: the consolidation arithmetic and the fused plan
+    at full size, to 1e-5 relative (heads 0 and 11 tracked in full by the oracle)."""
+    p = Pair(21, 12, 128, 1560, beta=0.3, dtype=torch.float32, seed=3, tracked_heads=[0, 11], device_gen=True)
+    for seg in range(12):
+        p.step(3)
+    p.check_entries()
+    p.check_memory()
+    rows = np.array([0, 1, 777, 2048, 4679])
+    p.check_attend(p.queries(4680, step=12), rows=rows)
+
+
 def test_wan13b_single_layer_full_size():
     """Wan-1.3B shape (H=12, D=128, N=1560, M=21, Lq=4680), the launch the bench times.
 
