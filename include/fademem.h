@@ -162,6 +162,30 @@ FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void *stream, 
 /* Forget every entry (count = 0, t = 0).  Enqueued on stream. */
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
 
+/* Bytes of library-owned device scratch used by fademem_consolidate_noalloc. */
+#define FADEMEM_NOALLOC_SCRATCH_BYTES 4096
+
+/* fademem_consolidate without any scratch in the caller's workspace and without
+ * any allocation (no cudaMalloc, cudaFree or allocating library call): the
+ * per-call working state (a copy of the entry table, the merge plan and the
+ * status word) lives in a file-scope device array of the library, of
+ * FADEMEM_NOALLOC_SCRATCH_BYTES bytes, that every GPU which loads the library
+ * holds until the process exits.  The paper has no counterpart: this serves
+ * callers that may not allocate device memory once they are running, such as
+ * plug-ins of a host framework that owns all device memory, or real-time loops
+ * that fix their memory at start-up.  The caller still passes the memory
+ * (workspace of fademem_create) and the inserted frames, as for
+ * fademem_consolidate, and the results are the same.
+ * The first call on each device looks up the array's device address with that
+ * device current (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  Every call shares the one array: calls that overlap on the
+ * GPU (other streams, other handles, other threads) race and must be
+ * serialised by the caller.  Nothing in the array needs clearing: each call
+ * overwrites it from the handle's workspace before use.  A handle whose entry
+ * table would not fit the array (budget above FADEMEM_MAX_BUDGET) is rejected
+ * with FADEMEM_ERR_UNSUPPORTED.  Other errors as fademem_consolidate. */
+FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void *stream);
+
 /* Release the handle (NULL-safe).  Does not free the caller's workspace. */
 FADEMEM_API void fademem_destroy(fademem_t h);
 

@@ -6,6 +6,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -321,6 +322,66 @@ FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
     h->pending[l].clear();
     h->pending_frames[l] = 0;
   }
+  return FADEMEM_OK;
+}
+
+}  // extern "C"
+
+// ---- Consolidation with library-owned scratch (fademem_consolidate_noalloc) ----
+namespace {
+
+// Working copy of one handle's DevState (entry table, merge plan, status word)
+// for fademem_consolidate_noalloc.  Host code must not pass this name to a
+// kernel: on the host it is only a stand-in; its device address comes from
+// cudaGetSymbolAddress, once per device.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[FADEMEM_NOALLOC_SCRATCH_BYTES];
+static_assert(sizeof(DevState) <= FADEMEM_NOALLOC_SCRATCH_BYTES, "DevState must fit the no-alloc scratch");
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+fademem_status noalloc_scratch(DevState** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(FADEMEM_ERR_UNSUPPORTED, "device %d out of range", dev);
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // with this device current
+    if (e != cudaSuccess) return cuda_fail(e, "looking up the no-alloc scratch");
+    g_scratch_addr[dev] = p;
+  }
+  *out = reinterpret_cast<DevState*>(g_scratch_addr[dev]);
+  return FADEMEM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (h->g.M + 1 > kMaxEntries)
+    return fail(FADEMEM_ERR_UNSUPPORTED, "budget %d does not fit the %d-byte no-alloc scratch", h->g.M,
+                FADEMEM_NOALLOC_SCRATCH_BYTES);
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  DevState* scratch = nullptr;
+  fademem_status s = noalloc_scratch(&scratch);
+  if (s != FADEMEM_OK) return s;
+  s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaMemcpyAsync(scratch, h->st, sizeof(DevState), cudaMemcpyDeviceToDevice, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "copying the entry table to the no-alloc scratch");
+  // Run the ordinary consolidation on the scratch copy, then copy the result back.
+  DevState* own = h->st;
+  h->st = scratch;
+  const fademem_status rs = fademem_consolidate(h, stream_);
+  h->st = own;
+  e = cudaMemcpyAsync(own, scratch, sizeof(DevState), cudaMemcpyDeviceToDevice, stream);
+  if (rs != FADEMEM_OK) return rs;
+  if (e != cudaSuccess) return cuda_fail(e, "copying the entry table back from the no-alloc scratch");
   return FADEMEM_OK;
 }
 
