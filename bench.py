@@ -279,53 +279,72 @@ def run_cuda(args):
         torch.distributed.destroy_process_group()
 
 
-def cpu_baseline(n_queries: int = 48):
-    """The fp64 oracle as it stands, on this host's cores, on a bounded sample of the workload.
+class OracleStep:
+    """The fp64 oracle, as it stands, stepping the same workload on this host's cores.
 
-    Sample: one full steady-state consolidation step (3 frames into a 21-entry
-    memory, all 12 heads, every token) plus attention for n_queries of the 4680
-    query rows over all 12 heads and 32,760 keys per head; the attention time is
-    scaled to the 4680 rows of one step.
+    The memory is warmed once (M + 3 frames: full budget, merging).  One step
+    inserts a segment's 3 frames (a full steady-state consolidation of all 12
+    heads and every token, timed) and attends a bounded sample of the 4680
+    query rows over all 12 heads and 32,760 keys per head (timed); the
+    attention time is scaled to the 4680 rows.  Frame generation is not timed.
     """
-    from oracle import OracleMemory, oracle_num_threads
-    from synth import KIND_K, KIND_V, HostAR1, host_queries
-    elems = N * H * D
-    mem = OracleMemory(M, BETA, anchor=True, elems=elems)
-    gk = HostAR1((N, H, D), 7, KIND_K)
-    gv = HostAR1((N, H, D), 7, KIND_V)
 
-    def frame(g):
+    def __init__(self, seed: int = 7):
+        from oracle import OracleMemory
+        from synth import KIND_K, KIND_V, HostAR1
+        self.mem = OracleMemory(M, BETA, anchor=True, elems=N * H * D)
+        self.gk = HostAR1((N, H, D), seed, KIND_K)
+        self.gv = HostAR1((N, H, D), seed, KIND_V)
+        self.seed = seed
+        self.steps = 0
+        for _ in range(M + 3):
+            self.mem.insert(self._frame(self.gk), self._frame(self.gv))
+
+    @staticmethod
+    def _frame(g):
         return torch.from_numpy(g.next()).to(torch.bfloat16).double().numpy()
-    for _ in range(M + 3):  # fill the budget and start merging
-        mem.insert(frame(gk), frame(gv))
-    new = [(frame(gk), frame(gv)) for _ in range(F)]
-    t0 = time.perf_counter()
-    for K, V in new:
-        mem.insert(K, V)
-    t_cons = time.perf_counter() - t0
-    Q = torch.from_numpy(host_queries((n_queries, H, D), 7)).to(torch.bfloat16).double().numpy()
-    t0 = time.perf_counter()
-    mem.attend(Q, N, H, D)
-    t_attn = time.perf_counter() - t0
-    step_s = t_cons + t_attn * (LQ / n_queries)
+
+    def step(self, n_queries: int):
+        from synth import host_queries
+        new = [(self._frame(self.gk), self._frame(self.gv)) for _ in range(F)]
+        Q = torch.from_numpy(host_queries((n_queries, H, D), self.seed, 0, self.steps)).to(
+            torch.bfloat16).double().numpy()
+        self.steps += 1
+        t0 = time.perf_counter()
+        for K, V in new:
+            self.mem.insert(K, V)
+        t_cons = time.perf_counter() - t0
+        t0 = time.perf_counter()
+        self.mem.attend(Q, N, H, D)
+        t_attn = time.perf_counter() - t0
+        return t_cons, t_attn, t_cons + t_attn * (LQ / n_queries)
+
+
+def _oracle_sample(n_queries: int) -> str:
+    return (f"fp64 C oracle: one full 3-frame consolidation (12 heads x 1560 tokens) + attention of "
+            f"{n_queries}/{LQ} query rows x {H} heads over {M * N} keys, scaled to {LQ} rows")
+
+
+def cpu_baseline(n_queries: int = 2340):
+    """One oracle step on a bounded sample (about 10 s of CPU work at the default)."""
+    from oracle import oracle_num_threads
+    o = OracleStep()
+    t_cons, t_attn, step_s = o.step(n_queries)
     return {"value": round(LQ / step_s, 3), "unit": "tokens/s", "cores": oracle_num_threads(), "kind": "oracle",
-            "sample": f"fp64 C oracle: one full 3-frame consolidation (all heads/tokens) + attention of "
-                      f"{n_queries}/{LQ} query rows x {H} heads over {M * N} keys, scaled to {LQ} rows",
-            "seconds_measured": round(t_cons + t_attn, 2)}
+            "sample": _oracle_sample(n_queries), "seconds_measured": round(t_cons + t_attn, 2)}
 
 
 def run_reference(args):
     """The oracle as the reference arm: each step a bounded sample of the same workload."""
+    from oracle import oracle_num_threads
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    times = []
-    base = None
-    for i in range(args.warmup + args.steps):
-        r = cpu_baseline(args.cpu_queries)
-        if i >= args.warmup:
-            times.append(LQ / r["value"])
-        base = r
+    nq = args.ref_queries
+    o = OracleStep()
+    for _ in range(args.warmup):
+        o.step(nq)
+    times = [o.step(nq)[2] for _ in range(args.steps)]
     step_s = statistics.mean(times)
     value = LQ / step_s
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws,
@@ -333,8 +352,8 @@ def run_reference(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (AR(1) K/V rho=0.9, N(0,1) Q)",
             "config": {"workload": WORKLOAD},
-            "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": base["cores"], "kind": "oracle",
-                             "sample": base["sample"]},
+            "cpu_baseline": {"value": round(value, 3), "unit": "tokens/s", "cores": oracle_num_threads(),
+                             "kind": "oracle", "sample": _oracle_sample(nq)},
             "e2e": {"value": round(value, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -346,7 +365,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-queries", type=int, default=48)
+    ap.add_argument("--cpu-queries", type=int, default=2340, help="query rows of the cpu_baseline sample")
+    ap.add_argument("--ref-queries", type=int, default=240, help="query rows per --impl reference step")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -3,19 +3,25 @@
 // tensor cores: per head, out = softmax(scale * Q K^T) V over all count*N
 // cached keys.
 //
-// One CTA computes one 128-query tile of one head:
-//   warp 4      TMA producer: Q tile once, then K/V tiles of 128 keys into a
-//               2-stage ring (128-byte swizzle, zero fill past the last key)
-//   warp 5      allocates 512 TMEM columns and issues tcgen05.mma:
-//               S_j = Q K_j^T into TMEM buffer j%2 (fp32), and after the
-//               softmax of tile j, O += P_j V_j into the TMEM accumulator
-//   warps 0-3   softmax, one thread per query row (= TMEM lane): load S_j,
-//               online softmax in the exp2 domain with a lazily updated
-//               reference maximum (O is rescaled only when the row maximum
-//               grows by more than 2^8), write P_j as bf16 into shared memory
-//               in the swizzled K-major layout, then the epilogue O / l.
-// S_{j+1} is computed while the softmax of tile j runs.  Every mbarrier wait
-// is bounded; on time-out the CTA records it in the status word and leaves.
+// One CTA computes one 128-query tile of one head, 352 threads:
+//   warp 8      TMA producer of Q (once) and of K tiles of 128 keys into a
+//               3-stage ring (128-byte swizzle, zero fill past the last key)
+//   warp 10     TMA producer of V tiles into a 2-stage ring, so a slow V slot
+//               never holds back the next K tile
+//   warp 9      allocates 512 TMEM columns and issues tcgen05.mma
+//   warps 0-7   two softmax groups of four warps; group g takes the key tiles
+//               j = g, g+2, ... with its own online-softmax state (m, l) and
+//               its own accumulator O_g in TMEM (one query row per thread =
+//               TMEM lane).  Per tile: load S_j, exp2-domain softmax with a
+//               lazily updated reference maximum (O_g is rescaled only when
+//               the row maximum grows by more than 2^8), write P_j as bf16
+//               pairs over S_j in TMEM.
+// P_j V_j reads P from TMEM (tcgen05.mma with the A operand in TMEM), so the
+// only shared-memory traffic per tile is Q and the K/V tiles.  While one group
+// runs its softmax, the tensor pipe runs the other group's P·V and next Q·K^T,
+// so the tensor pipe and the exponential unit overlap.  The epilogue combines
+// (O_0, m_0, l_0) and (O_1, m_1, l_1) row by row.  Every mbarrier wait is
+// bounded; on time-out the CTA records it in the status word and leaves.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdio.h>
@@ -28,22 +34,30 @@ namespace {
 constexpr int kBM = 128;        // query rows per tile (TMEM lanes)
 constexpr int kBN = 128;        // keys per tile
 constexpr int kHD = 128;        // head dimension
-constexpr int kStages = 2;
-constexpr int kThreads = 192;
+constexpr int kSoftmaxThreads = 256;  // two groups of four warps
+constexpr int kWarpTma = 8;    // Q and K producer
+constexpr int kWarpMma = 9;
+constexpr int kWarpTmaV = 10;  // V producer
+constexpr int kThreads = 352;
+constexpr int kKStages = 3;
+constexpr int kVStages = 2;
 constexpr uint32_t kHalfBytes = kBM * 64 * 2;   // 128 rows x 64 bf16 (one swizzle-128B panel)
 constexpr uint32_t kTileBytes = 2 * kHalfBytes; // 128 rows x 128 bf16
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kTileBytes;
-constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
-constexpr uint32_t kOffP = kOffV + kStages * kTileBytes;
-constexpr uint32_t kOffBar = kOffP + kTileBytes;
-constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;  // barriers + alignment slack
+constexpr uint32_t kOffV = kOffK + kKStages * kTileBytes;
+constexpr uint32_t kOffBar = kOffV + kVStages * kTileBytes;
+constexpr uint32_t kOffML = kOffBar + 256;           // per-row (m, l) of both groups
+constexpr uint32_t kSmemBytes = kOffML + 4 * kBM * 4 + 1024;  // + alignment slack
 constexpr uint32_t kTmemCols = 512;
+// TMEM columns: S_0 [0,128), S_1 [128,256) fp32 (P_g overwrites the first 64
+// columns of S_g as bf16 pairs); O_0 [256,384), O_1 [384,512) fp32.
+constexpr uint32_t kColO = 256;
 constexpr long long kWaitLimitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 // Barrier indices (8 bytes each at kOffBar).
-enum { BAR_Q = 0, BAR_KFULL = 1, BAR_VFULL = 3, BAR_KEMPTY = 5, BAR_VEMPTY = 7, BAR_SFULL = 9, BAR_PFULL = 11,
-       BAR_ODONE = 12, BAR_FINAL = 13, BAR_COUNT = 14 };
+enum { BAR_Q = 0, BAR_KFULL = 1, BAR_KEMPTY = 4, BAR_VFULL = 7, BAR_VEMPTY = 9, BAR_SFULL = 11, BAR_PFULL = 13,
+       BAR_FINAL = 15, BAR_COUNT = 16 };
 
 struct AttnParams {
   CUtensorMap tmQ;   // [Lq][H][D]  dims (D, H, Lq), box (64, 1, 128)
@@ -111,6 +125,16 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint
       "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Same, with the A operand in TMEM (rows on lanes, two 16-bit elements per column).
+__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                             uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
@@ -133,6 +157,13 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
       "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
       FM_W8(0), FM_W8(8), FM_W8(16), FM_W8(24)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16};" ::"r"(taddr),
+      FM_W8(0), FM_W8(8)
       : "memory");
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
@@ -172,6 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = sbase + kOffBar;
   auto bar = [&](int i) { return bar0 + 8u * i; };
+  float* s_ml = reinterpret_cast<float*>(smem + kOffML);  // [2 groups][2 (m, l)][128 rows]
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
 
@@ -183,26 +215,29 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   if (threadIdx.x == 0) {
     s_abort = 0;
     mbar_init(bar(BAR_Q), 1);
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       mbar_init(bar(BAR_KFULL + s), 1);
-      mbar_init(bar(BAR_VFULL + s), 1);
       mbar_init(bar(BAR_KEMPTY + s), 1);
-      mbar_init(bar(BAR_VEMPTY + s), 1);
-      mbar_init(bar(BAR_SFULL + s), 1);
     }
-    mbar_init(bar(BAR_PFULL), 128);
-    mbar_init(bar(BAR_ODONE), 1);
+    for (int s = 0; s < kVStages; ++s) {
+      mbar_init(bar(BAR_VFULL + s), 1);
+      mbar_init(bar(BAR_VEMPTY + s), 1);
+    }
+    for (int g = 0; g < 2; ++g) {
+      mbar_init(bar(BAR_SFULL + g), 1);
+      mbar_init(bar(BAR_PFULL + g), 128);
+    }
     mbar_init(bar(BAR_FINAL), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
                  "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  if (warp == 4 && lane == 0) {
+  if (warp == kWarpTma && lane == 0) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmQ)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmV)) : "memory");
@@ -210,6 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // Launched as a programmatic dependent: the set-up above overlaps the
+  // previous kernel; nothing in global memory is touched before this wait.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const uint32_t tmem = s_tmem;
   volatile int* abort_flag = &s_abort;
   auto fail = [&]() {
@@ -217,95 +255,118 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
     atomicOr(p.status, kStatusTimeout);
   };
 
-  if (warp == 4) {
-    // ---------------- TMA producer ----------------
+  if (warp == kWarpTma) {
+    // ---------------- TMA producer of Q (once) and K_j into stage j%3 ----------------
     if (lane == 0) {
       const uint32_t sQ = sbase + kOffQ;
       mbar_expect_tx(bar(BAR_Q), kTileBytes);
       tma_load_3d(sQ, &p.tmQ, bar(BAR_Q), 0, h, q0);
       tma_load_3d(sQ + kHalfBytes, &p.tmQ, bar(BAR_Q), 64, h, q0);
       for (int j = 0; j < n_tiles; ++j) {
-        const int s = j % kStages;
-        const uint32_t par = ((j / kStages) & 1) ^ 1;
-        if (j >= kStages && !mbar_wait(bar(BAR_KEMPTY + s), par, abort_flag)) { fail(); break; }
+        const int s = j % kKStages;
+        if (j >= kKStages && !mbar_wait(bar(BAR_KEMPTY + s), ((j / kKStages) & 1) ^ 1, abort_flag)) {
+          fail();
+          break;
+        }
         const uint32_t sK = sbase + kOffK + s * kTileBytes;
         mbar_expect_tx(bar(BAR_KFULL + s), kTileBytes);
         tma_load_3d(sK, &p.tmK, bar(BAR_KFULL + s), 0, j * kBN, h);
         tma_load_3d(sK + kHalfBytes, &p.tmK, bar(BAR_KFULL + s), 64, j * kBN, h);
-        if (j >= kStages && !mbar_wait(bar(BAR_VEMPTY + s), par, abort_flag)) { fail(); break; }
+      }
+    }
+  } else if (warp == kWarpTmaV) {
+    // ---------------- TMA producer of V_j into stage j%2 (independent of the K ring) ----------------
+    if (lane == 0) {
+      for (int j = 0; j < n_tiles; ++j) {
+        const int s = j % kVStages;
+        if (j >= kVStages && !mbar_wait(bar(BAR_VEMPTY + s), ((j / kVStages) & 1) ^ 1, abort_flag)) {
+          fail();
+          break;
+        }
         const uint32_t sV = sbase + kOffV + s * kTileBytes;
         mbar_expect_tx(bar(BAR_VFULL + s), kTileBytes);
         tma_load_3d(sV, &p.tmV, bar(BAR_VFULL + s), 0, j * kBN, h);
         tma_load_3d(sV + kHalfBytes, &p.tmV, bar(BAR_VFULL + s), 64, j * kBN, h);
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kWarpMma) {
     // ---------------- MMA issuer ----------------
+    // Tile j belongs to softmax group j%2: S_j goes to TMEM buffer j%2, the group
+    // writes P_j over the first 64 columns of that buffer, and P_j V_j goes to the
+    // group's own accumulator O_{j%2}.  The tensor pipe runs tcgen05.mma in issue
+    // order, so issuing S_{j+2} after P_j V_j never overwrites P_j too early.
     if (lane == 0) {
       constexpr uint32_t idesc_qk = make_idesc(kBM, kBN, 0);
       constexpr uint32_t idesc_pv = make_idesc(kBM, kHD, 1);
-      const uint32_t sQ = sbase + kOffQ, sP = sbase + kOffP;
-      const uint32_t tO = tmem + 256;
+      // Descriptors are built once per operand buffer and advanced along K by adding
+      // (byte offset >> 4) to the start-address field: the issuing thread must not
+      // spend a dependent integer chain per MMA, or issue (not the tensor pipe) limits.
+      const uint64_t dQ = sw128_desc(sbase + kOffQ, 16, 1024);
+      auto issue_qk = [&](int j) -> bool {
+        const int s = j % kKStages;
+        if (!mbar_wait(bar(BAR_KFULL + s), (j / kKStages) & 1, abort_flag)) return false;
+        tc_fence_after();
+        const uint64_t dK = sw128_desc(sbase + kOffK + s * kTileBytes, 16, 1024);
+        const uint32_t tS = tmem + (j & 1) * kBN;
+#pragma unroll
+        for (int kk = 0; kk < kHD / 16; ++kk) {
+          const uint64_t off = ((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4;
+          umma_bf16(tS, dQ + off, dK + off, idesc_qk, kk > 0);
+        }
+        umma_commit(bar(BAR_SFULL + (j & 1)));
+        umma_commit(bar(BAR_KEMPTY + s));
+        return true;
+      };
       bool ok = mbar_wait(bar(BAR_Q), 0, abort_flag);
       if (!ok) fail();
       tc_fence_after();
-      for (int j = 0; ok && j <= n_tiles; ++j) {
-        if (j < n_tiles) {
-          const int s = j % kStages;
-          if (!mbar_wait(bar(BAR_KFULL + s), (j / kStages) & 1, abort_flag)) { fail(); break; }
-          tc_fence_after();
-          const uint32_t sK = sbase + kOffK + s * kTileBytes;
-          const uint32_t tS = tmem + (j & 1) * 128;
+      for (int j = 0; ok && j < 2 && j < n_tiles; ++j)
+        if (!issue_qk(j)) { fail(); ok = false; }
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int g = j & 1, s = j % kVStages;
+        if (!mbar_wait(bar(BAR_PFULL + g), (j >> 1) & 1, abort_flag)) { fail(); break; }
+        if (!mbar_wait(bar(BAR_VFULL + s), (j / kVStages) & 1, abort_flag)) { fail(); break; }
+        tc_fence_after();
+        const uint64_t dV = sw128_desc(sbase + kOffV + s * kTileBytes, kHalfBytes, 1024);
+        const uint32_t tP = tmem + g * kBN;
+        const uint32_t tO = tmem + kColO + g * kHD;
 #pragma unroll
-          for (int kk = 0; kk < kHD / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-            umma_bf16(tS, sw128_desc(sQ + off, 16, 1024), sw128_desc(sK + off, 16, 1024), idesc_qk, kk > 0);
-          }
-          umma_commit(bar(BAR_SFULL + (j & 1)));
-          umma_commit(bar(BAR_KEMPTY + s));
+        for (int kk = 0; kk < kBN / 16; ++kk) {
+          umma_bf16_ts(tO, tP + kk * 8, dV + (uint64_t)(kk * (2048 >> 4)), idesc_pv, (j >= 2 || kk > 0) ? 1u : 0u);
         }
-        if (j >= 1) {
-          const int jj = j - 1;
-          const int s = jj % kStages;
-          if (!mbar_wait(bar(BAR_PFULL), jj & 1, abort_flag)) { fail(); break; }
-          if (!mbar_wait(bar(BAR_VFULL + s), (jj / kStages) & 1, abort_flag)) { fail(); break; }
-          tc_fence_after();
-          const uint32_t sV = sbase + kOffV + s * kTileBytes;
-#pragma unroll
-          for (int kk = 0; kk < kBN / 16; ++kk) {
-            const uint32_t offp = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-            umma_bf16(tO, sw128_desc(sP + offp, 16, 1024), sw128_desc(sV + kk * 2048, kHalfBytes, 1024), idesc_pv,
-                      (jj > 0 || kk > 0) ? 1u : 0u);
-          }
-          umma_commit(bar(BAR_ODONE));
-          umma_commit(bar(BAR_VEMPTY + s));
-        }
+        umma_commit(bar(BAR_VEMPTY + s));
+        if (j + 2 < n_tiles && !issue_qk(j + 2)) { fail(); break; }
       }
       // Drain: every MMA issued above has completed once this barrier flips.
       umma_commit(bar(BAR_FINAL));
       if (!mbar_wait(bar(BAR_FINAL), 0, abort_flag) && !*abort_flag) fail();
     }
   } else {
-    // ---------------- softmax + epilogue (warps 0-3, one query row per thread) ----------------
-    const int row = warp * 32 + lane;
-    const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-    const uint32_t tO = tmem + 256 + lane_off;
-    uint8_t* sP = smem + kOffP;
+    // ---------------- softmax groups 0/1 (warps 0-3 / 4-7), one query row per thread ----------------
+    const int grp = warp >> 2;
+    const int row = (warp & 3) * 32 + lane;
+    const uint32_t lane_off = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t tS = tmem + grp * kBN + lane_off;
+    const uint32_t tO = tmem + kColO + grp * kHD + lane_off;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
-    for (int j = 0; j < n_tiles; ++j) {
-      if (!mbar_wait(bar(BAR_SFULL + (j & 1)), (j >> 1) & 1, abort_flag)) { fail(); ok = false; break; }
+    for (int j = grp; j < n_tiles; j += 2) {
+      if (!mbar_wait(bar(BAR_SFULL + grp), (j >> 1) & 1, abort_flag)) { fail(); ok = false; break; }
       tc_fence_after();
       float sv[kBN];
       {
-        const uint32_t tS = tmem + (j & 1) * 128 + lane_off;
+        uint32_t r0[32], r1[32], r2[32], r3[32];
+        tmem_ld32(tS, r0);
+        tmem_ld32(tS + 32, r1);
+        tmem_ld32(tS + 64, r2);
+        tmem_ld32(tS + 96, r3);
+        tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < kBN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(tS + c * 32, r);
-          tmem_ld_wait();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) sv[c * 32 + i] = __uint_as_float(r[i]);
+        for (int i = 0; i < 32; ++i) {
+          sv[i] = __uint_as_float(r0[i]);
+          sv[32 + i] = __uint_as_float(r1[i]);
+          sv[64 + i] = __uint_as_float(r2[i]);
+          sv[96 + i] = __uint_as_float(r3[i]);
         }
       }
       if (j == n_tiles - 1) {
@@ -314,75 +375,93 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         for (int c = 0; c < kBN; ++c)
           if (c >= valid) sv[c] = -INFINITY;
       }
-      float mt = sv[0];
+      float mx[8];
 #pragma unroll
-      for (int c = 1; c < kBN; ++c) mt = fmaxf(mt, sv[c]);
-      mt *= p.scale_log2;
+      for (int k = 0; k < 8; ++k) mx[k] = sv[k];
+#pragma unroll
+      for (int c = 8; c < kBN; c += 8)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], sv[c + k]);
+      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * p.scale_log2;
       // Lazy reference maximum: move it only when the tile exceeds it by > 8 (2^8 headroom).
       const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
       const float m_new = move ? fmaxf(mt, m_run) : m_run;
-      const float alpha = ex2(m_run - m_new);  // 0 on the first tile, 1 if unchanged
-      float rs = 0.f;
-      uint32_t pk[kBN / 2];
+      const float alpha = ex2(m_run - m_new);  // 0 on the group's first tile, 1 if unchanged
+      float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
-      for (int c = 0; c < kBN; c += 2) {
-        const float e0 = ex2(fmaf(sv[c], p.scale_log2, -m_new));
-        const float e1 = ex2(fmaf(sv[c + 1], p.scale_log2, -m_new));
-        rs += e0 + e1;
-        pk[c / 2] = pack_bf16(e0, e1);
-      }
-      l_run = l_run * alpha + rs;
-      m_run = m_new;
-      if (j > 0) {
-        // PV of tile j-1 must be done: P is overwritten and O may be rescaled.
-        if (!mbar_wait(bar(BAR_ODONE), (j - 1) & 1, abort_flag)) { fail(); ok = false; break; }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, move)) {
+      for (int qtr = 0; qtr < 4; ++qtr) {
+        uint32_t pk[16];
 #pragma unroll
-          for (int c = 0; c < kHD / 32; ++c) {
-            uint32_t r[32];
-            tmem_ld32(tO + c * 32, r);
-            tmem_ld_wait();
-#pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
-            tmem_st32(tO + c * 32, r);
-          }
-          tmem_st_wait();
+        for (int c = 0; c < 32; c += 2) {
+          const float e0 = ex2(fmaf(sv[32 * qtr + c], p.scale_log2, -m_new));
+          const float e1 = ex2(fmaf(sv[32 * qtr + c + 1], p.scale_log2, -m_new));
+          rs0 += e0;
+          rs1 += e1;
+          pk[c / 2] = pack_bf16(e0, e1);
         }
+        tmem_st16(tS + qtr * 16, pk);  // P over the first 64 columns of the S buffer
       }
-      // P row -> shared memory, K-major with 128-byte swizzle (16-byte chunk c of
-      // row r lands at chunk c ^ (r % 8) of that row's 128-byte line).
-#pragma unroll
-      for (int c = 0; c < kBN / 8; ++c) {
-        const uint32_t off = (c >> 3) * kHalfBytes + row * 128 + ((((c & 7) ^ (row & 7))) << 4);
-        *reinterpret_cast<uint4*>(sP + off) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-      }
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      tc_fence_before();
-      mbar_arrive(bar(BAR_PFULL));
-    }
-    if (ok && n_tiles > 0) {
-      if (!mbar_wait(bar(BAR_ODONE), (n_tiles - 1) & 1, abort_flag)) {
-        fail();
-      } else {
-        tc_fence_after();
-        const float inv = 1.f / l_run;
-        const int q = q0 + row;
-        __nv_bfloat16* orow = p.out + ((size_t)q * p.H + h) * kHD;
+      l_run = l_run * alpha + (rs0 + rs1);
+      m_run = m_new;
+      if (j >= 2 && __any_sync(0xffffffffu, move)) {
+        // Rescale O_grp before P_j V_j accumulates into it.  Its last update
+        // (P_{j-2} V_{j-2}) was issued before S_j, so it is complete once S_j is.
 #pragma unroll
         for (int c = 0; c < kHD / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(tO + c * 32, r);
           tmem_ld_wait();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+          tmem_st32(tO + c * 32, r);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(bar(BAR_PFULL + grp));
+    }
+    // ---------------- epilogue: combine the two groups' (O, m, l) ----------------
+    s_ml[(grp * 2 + 0) * kBM + row] = m_run;
+    s_ml[(grp * 2 + 1) * kBM + row] = l_run;
+    asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+    if (ok && !*abort_flag) {
+      if (!mbar_wait(bar(BAR_FINAL), 0, abort_flag)) {
+        fail();
+      } else {
+        tc_fence_after();
+        const float m0 = s_ml[0 * kBM + row], l0 = s_ml[1 * kBM + row];
+        const float m1 = s_ml[2 * kBM + row], l1 = s_ml[3 * kBM + row];
+        const bool has1 = n_tiles > 1;
+        const float m = has1 ? fmaxf(m0, m1) : m0;
+        const float f0 = ex2(m0 - m);
+        const float f1 = has1 ? ex2(m1 - m) : 0.f;
+        const float inv = 1.f / (l0 * f0 + l1 * f1);
+        const float a0 = f0 * inv, a1 = f1 * inv;
+        const int q = q0 + row;
+        __nv_bfloat16* orow = p.out + ((size_t)q * p.H + h) * kHD;
+        const uint32_t tO0 = tmem + kColO + lane_off;
+        const uint32_t tO1 = tmem + kColO + kHD + lane_off;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const int col = grp * 64 + c * 32;  // this group writes columns [64 grp, 64 grp + 64)
+          uint32_t r0[32], r1[32];
+          tmem_ld32(tO0 + col, r0);
+          if (has1) tmem_ld32(tO1 + col, r1);
+          tmem_ld_wait();
           if (q < p.Lq) {
 #pragma unroll
             for (int i = 0; i < 32; i += 8) {
+              float o[8];
+#pragma unroll
+              for (int e = 0; e < 8; ++e)
+                o[e] = __uint_as_float(r0[i + e]) * a0 + (has1 ? __uint_as_float(r1[i + e]) * a1 : 0.f);
               uint4 v;
-              v.x = pack_bf16(__uint_as_float(r[i]) * inv, __uint_as_float(r[i + 1]) * inv);
-              v.y = pack_bf16(__uint_as_float(r[i + 2]) * inv, __uint_as_float(r[i + 3]) * inv);
-              v.z = pack_bf16(__uint_as_float(r[i + 4]) * inv, __uint_as_float(r[i + 5]) * inv);
-              v.w = pack_bf16(__uint_as_float(r[i + 6]) * inv, __uint_as_float(r[i + 7]) * inv);
-              *reinterpret_cast<uint4*>(orow + c * 32 + i) = v;
+              v.x = pack_bf16(o[0], o[1]);
+              v.y = pack_bf16(o[2], o[3]);
+              v.z = pack_bf16(o[4], o[5]);
+              v.w = pack_bf16(o[6], o[7]);
+              *reinterpret_cast<uint4*>(orow + col + i) = v;
             }
           }
         }
@@ -392,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
@@ -462,9 +541,17 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
   prm.H = g.H;
   prm.scale_log2 = scale * 1.4426950408889634f;
   prm.status = status;
-  dim3 grid((Lq + kBM - 1) / kBM, g.H);
-  attend_tc_kernel<<<grid, kThreads, kSmemBytes, stream>>>(prm);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((Lq + kBM - 1) / kBM, g.H);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attend_tc_kernel, prm);
 }
 
 }  // namespace fademem

@@ -32,20 +32,52 @@ __device__ __forceinline__ double warp_u(double d, double beta) {
   return pow(d, beta);
 }
 
+// fp32 estimate of u(d) and a bound on its error.  powf is accurate to a few
+// ulp and beta rounded to fp32 moves d^beta by under beta * 2^-24 * ln(d)
+// relative, so 2^-16 relative (about 100x the worst case) is a safe bound.
+__device__ __forceinline__ float warp_u32(float d, float beta) {
+  if (beta == 1.0f) return d;
+  return powf(d, beta);
+}
+constexpr float kU32RelErr = 1.0f / 65536.0f;
+
 struct SchedShared {
   int slot[kMaxEntries];
   long long first[kMaxEntries];
   long long span[kMaxEntries];
-  double mu[kMaxEntries];
+  long long mu2[kMaxEntries];  // 2*mu: mu is always a half-integer (midpoint of a contiguous span)
   int natoms[kMaxEntries];
   int ref[kMaxEntries][kMaxPassFrames + 1];
-  double w[kMaxEntries][kMaxPassFrames + 1];
+  float w[kMaxEntries][kMaxPassFrames + 1];
+  float u32[kMaxEntries];
+  int dest[kMaxEntries];     // plan: destination index of a changed entry, -1 if unchanged
+  int src0[kMaxEntries];     // plan: first source index of a changed entry
 };
 
+// Lowest (value, index) over the warp.
+__device__ __forceinline__ void warp_argmin(double& v, int& i) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const double ov = __shfl_xor_sync(0xffffffffu, v, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, i, off);
+    if (ov < v || (ov == v && oi < i)) { v = ov; i = oi; }
+  }
+}
+
+// Algorithm S1 for `frames` units, one warp.  The pair chosen for each frame
+// is exactly the argmin (lowest index on ties) of the fp64 gaps
+// |warp_u(t - mu_{i+1}) - warp_u(t - mu_i)|: every pair is first scored in
+// fp32 with an error bound E_i, and only pairs whose fp32 interval can reach
+// the smallest upper bound U = min_k (g32_k + E_k) are scored again in fp64.
+// A pair outside that set has a true gap above the true minimum by more than
+// the fp64 rounding, so it cannot be the fp64 argmin either.
 __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, int M, double beta, int anchor,
                                                       int op, int expected_count) {
   __shared__ SchedShared s;
   const int lane = threadIdx.x;
+  // The consolidation kernel launched after this one may start now: it waits
+  // for this grid's completion before it reads the plan.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   DevMeta& m = st->meta;
   int count = m.count;
   if (count != expected_count || count < 0 || count > M) {
@@ -54,14 +86,15 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     return;
   }
   const long long t0 = m.t_next;
+  const float beta32 = (float)beta;
   for (int i = lane; i < count; i += 32) {
     s.slot[i] = m.slot[i];
     s.first[i] = m.first[i];
     s.span[i] = m.span[i];
-    s.mu[i] = m.mu[i];
+    s.mu2[i] = __double2ll_rn(2.0 * m.mu[i]);
     s.natoms[i] = 1;
     s.ref[i][0] = m.slot[i];  // content: the block now stored in its own slot
-    s.w[i][0] = 1.0;
+    s.w[i][0] = 1.0f;
   }
   __syncwarp();
   int merged[kMaxPassFrames];
@@ -70,10 +103,10 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     if (lane == 0) {  // Append (K_t, V_t, t, 1)
       s.first[count] = t;
       s.span[count] = 1;
-      s.mu[count] = (double)t;
+      s.mu2[count] = 2 * t;
       s.natoms[count] = 1;
       s.ref[count][0] = -(f + 1);
-      s.w[count][0] = 1.0;
+      s.w[count][0] = 1.0f;
       s.slot[count] = count;  // next free slot unless a merge frees one below
     }
     count += 1;
@@ -83,82 +116,149 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
 
     // Eligible pairs: (i, i+1) for i <= count-3 (the pair holding the newest is excluded).
     const int npairs = count - 2;
-    double best = INFINITY;
-    int bi = 0x7fffffff;
+    for (int i = lane; i <= npairs; i += 32) s.u32[i] = warp_u32(0.5f * (float)(2 * t - s.mu2[i]), beta32);
+    __syncwarp();
+    float ub = INFINITY;
     for (int i = lane; i < npairs; i += 32) {
-      const double g = fabs(warp_u((double)t - s.mu[i + 1], beta) - warp_u((double)t - s.mu[i], beta));
-      if (g < best) { best = g; bi = i; }
+      const float a = s.u32[i], b = s.u32[i + 1];
+      ub = fminf(ub, fabsf(b - a) + kU32RelErr * (a + b));
     }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const double og = __shfl_xor_sync(0xffffffffu, best, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-      if (og < best || (og == best && oi < bi)) { best = og; bi = oi; }
+    for (int off = 16; off > 0; off >>= 1) ub = fminf(ub, __shfl_xor_sync(0xffffffffu, ub, off));
+    double best = INFINITY;
+    int bi = 0x7fffffff, ncand = 0;
+    for (int i0 = 0; i0 < npairs; i0 += 32) {
+      const int i = i0 + lane;
+      bool cand = false;
+      if (i < npairs) {
+        const float a = s.u32[i], b = s.u32[i + 1];
+        cand = fabsf(b - a) - kU32RelErr * (a + b) <= ub;
+      }
+      const unsigned mask = __ballot_sync(0xffffffffu, cand);
+      ncand += __popc(mask);
+      if (cand && i < bi) bi = i;  // lowest-index candidate of this lane
+    }
+    if (ncand > 1) {  // several pairs may be the minimum: decide in fp64
+      bi = 0x7fffffff;
+      for (int i = lane; i < npairs; i += 32) {
+        const float a = s.u32[i], b = s.u32[i + 1];
+        if (fabsf(b - a) - kU32RelErr * (a + b) <= ub) {
+          const double g = fabs(warp_u(0.5 * (double)(2 * t - s.mu2[i + 1]), beta) -
+                                warp_u(0.5 * (double)(2 * t - s.mu2[i]), beta));
+          if (g < best) { best = g; bi = i; }
+        }
+      }
+      warp_argmin(best, bi);
+    } else {
+      double v = 0.0;
+      warp_argmin(v, bi);  // the single candidate
     }
     const int j = bi;
     merged[f] = j;
     if (lane == 0) {
       const long long sa = s.span[j], sb = s.span[j + 1];
       const long long s_new = sa + sb;
-      double mu_new;
+      long long mu2_new;
       if (anchor && j == 0) {
-        mu_new = 0.0;  // the anchor keeps its block and centre
+        mu2_new = 0;  // the anchor keeps its block and centre
       } else {
-        mu_new = ((double)sa * s.mu[j] + (double)sb * s.mu[j + 1]) / (double)s_new;
-        double wa = 1.0, wb = 1.0;
+        // mu_new = (s_j mu_j + s_{j+1} mu_{j+1}) / s_new, exactly, on 2*mu (the
+        // span-weighted centre of two adjacent contiguous runs is a half-integer).
+        mu2_new = (sa * s.mu2[j] + sb * s.mu2[j + 1]) / s_new;
+        float wa = 1.0f, wb = 1.0f;
         if (op == FADEMEM_MERGE_WEIGHTED) {
-          wa = sqrt((double)sa) / (sqrt((double)sa) + sqrt((double)sb));
-          wb = 1.0 - wa;
+          wa = sqrtf((float)sa) / (sqrtf((float)sa) + sqrtf((float)sb));
+          wb = 1.0f - wa;
         } else if (op == FADEMEM_MERGE_AVERAGE) {
-          wa = 0.5; wb = 0.5;
+          wa = 0.5f; wb = 0.5f;
         } else if (op == FADEMEM_MERGE_SELECT_NEAREST) {
-          wa = 0.0; wb = 1.0;
+          wa = 0.0f; wb = 1.0f;
         }
         int n = 0;
         int ref[kMaxPassFrames + 1];
-        double w[kMaxPassFrames + 1];
+        float w[kMaxPassFrames + 1];
         for (int k = 0; k < s.natoms[j]; ++k)
-          if (wa != 0.0) { ref[n] = s.ref[j][k]; w[n] = s.w[j][k] * wa; ++n; }
+          if (wa != 0.0f) { ref[n] = s.ref[j][k]; w[n] = s.w[j][k] * wa; ++n; }
         for (int k = 0; k < s.natoms[j + 1]; ++k)
-          if (wb != 0.0 && n <= kMaxPassFrames) { ref[n] = s.ref[j + 1][k]; w[n] = s.w[j + 1][k] * wb; ++n; }
+          if (wb != 0.0f && n <= kMaxPassFrames) { ref[n] = s.ref[j + 1][k]; w[n] = s.w[j + 1][k] * wb; ++n; }
         s.natoms[j] = n;
         for (int k = 0; k < n; ++k) { s.ref[j][k] = ref[k]; s.w[j][k] = w[k]; }
       }
       s.span[j] = s_new;
-      s.mu[j] = mu_new;
-      const int freed = s.slot[j + 1];
-      for (int i = j + 1; i < count - 1; ++i) {
-        s.slot[i] = s.slot[i + 1];
-        s.first[i] = s.first[i + 1];
-        s.span[i] = s.span[i + 1];
-        s.mu[i] = s.mu[i + 1];
-        s.natoms[i] = s.natoms[i + 1];
-        for (int k = 0; k < s.natoms[i]; ++k) { s.ref[i][k] = s.ref[i + 1][k]; s.w[i][k] = s.w[i + 1][k]; }
-      }
-      s.slot[count - 2] = freed;  // the newest entry takes m_{j+1}'s slot
+      s.mu2[j] = mu2_new;
     }
+    const int freed = s.slot[j + 1];
+    __syncwarp();
+    // Remove m_{j+1}: entries j+2 .. count-1 move down one place (lane-parallel).
+    for (int base = j + 1; base < count - 1; base += 32) {
+      const int i = base + lane;
+      int slot = 0, na = 0;
+      long long first = 0, span = 0, mu2 = 0;
+      int ref[kMaxPassFrames + 1];
+      float w[kMaxPassFrames + 1];
+      const bool mv = i < count - 1;
+      if (mv) {
+        slot = s.slot[i + 1]; first = s.first[i + 1]; span = s.span[i + 1]; mu2 = s.mu2[i + 1];
+        na = s.natoms[i + 1];
+#pragma unroll
+        for (int k = 0; k <= kMaxPassFrames; ++k) { ref[k] = s.ref[i + 1][k]; w[k] = s.w[i + 1][k]; }
+      }
+      __syncwarp();
+      if (mv) {
+        s.slot[i] = slot; s.first[i] = first; s.span[i] = span; s.mu2[i] = mu2; s.natoms[i] = na;
+#pragma unroll
+        for (int k = 0; k <= kMaxPassFrames; ++k) { s.ref[i][k] = ref[k]; s.w[i][k] = w[k]; }
+      }
+      __syncwarp();
+    }
+    if (lane == 0) s.slot[count - 2] = freed;  // the newest entry takes m_{j+1}'s slot
     count -= 1;
     __syncwarp();
   }
 
-  if (lane == 0) {
-    DevPlan& p = st->plan;
-    int ns = 0, nd = 0;
-    bool overflow = false;
-    for (int i = 0; i < count; ++i) {
-      const bool same = s.natoms[i] == 1 && s.ref[i][0] == s.slot[i] && s.w[i][0] == 1.0;
-      if (same) continue;
-      if (nd >= kMaxDest || ns + s.natoms[i] > kMaxSrc) { overflow = true; break; }
-      p.dest_slot[nd] = s.slot[i];
-      for (int k = 0; k < s.natoms[i]; ++k) {
-        p.src_ref[ns] = s.ref[i][k];
-        p.src_w[ns] = (float)s.w[i][k];
-        p.src_dest[ns] = nd;
-        ++ns;
-      }
-      ++nd;
+  // Merge plan: every entry whose block changed becomes a destination; its
+  // sources are stored contiguously, in entry order (lane-parallel prefix sums).
+  int nd = 0, ns = 0;
+  for (int base = 0; base < count; base += 32) {
+    const int i = base + lane;
+    bool changed = false;
+    int na = 0;
+    if (i < count) {
+      changed = !(s.natoms[i] == 1 && s.ref[i][0] == s.slot[i] && s.w[i][0] == 1.0f);
+      na = changed ? s.natoms[i] : 0;
     }
-    if (overflow) { ns = 0; nd = 0; atomicOr(&st->status, kStatusPlanOverflow); }
+    const unsigned cm = __ballot_sync(0xffffffffu, changed);
+    int incl = na;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int o = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += o;
+    }
+    if (i < count) {
+      s.dest[i] = changed ? nd + __popc(cm & ((1u << lane) - 1u)) : -1;
+      s.src0[i] = ns + incl - na;
+    }
+    nd += __popc(cm);
+    ns += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  __syncwarp();
+  DevPlan& p = st->plan;
+  const bool overflow = nd > kMaxDest || ns > kMaxSrc;
+  if (!overflow) {
+    for (int i = lane; i < count; i += 32) {
+      const int d = s.dest[i];
+      if (d < 0) continue;
+      p.dest_slot[d] = s.slot[i];
+      for (int k = 0; k < s.natoms[i]; ++k) {
+        const int q = s.src0[i] + k;
+        p.src_ref[q] = s.ref[i][k];
+        p.src_w[q] = s.w[i][k];
+        p.src_dest[q] = d;
+      }
+    }
+  }
+  if (lane == 0) {
+    if (overflow) { nd = 0; ns = 0; atomicOr(&st->status, kStatusPlanOverflow); }
     p.n_src = ns;
     p.n_dest = nd;
     p.frames = frames;
@@ -171,7 +271,7 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     m.slot[i] = s.slot[i];
     m.first[i] = s.first[i];
     m.span[i] = s.span[i];
-    m.mu[i] = s.mu[i];
+    m.mu[i] = 0.5 * (double)s.mu2[i];
   }
 }
 
@@ -226,6 +326,9 @@ __global__ void __launch_bounds__(256) consolidate_kernel(const __grid_constant_
   __shared__ int s_ref[kMaxSrc], s_dest[kMaxSrc], s_dslot[kMaxDest];
   __shared__ float s_w[kMaxSrc];
   __shared__ int s_ns;
+  // Launched as a programmatic dependent of the schedule kernel: wait for it
+  // (and every earlier grid of the stream) before reading any global memory.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const DevPlan& p = a.st->plan;
   if (threadIdx.x < kMaxSrc) {
     s_ref[threadIdx.x] = p.src_ref[threadIdx.x];
@@ -317,14 +420,22 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   if (bx < 1) bx = 1;
   dim3 grid(bx, g.L * 2 * g.H);
   const bool mx = op == FADEMEM_MERGE_MAX_POOL;
-  if (g.dtype == FADEMEM_BF16) {
-    if (mx) consolidate_kernel<__nv_bfloat16, true><<<grid, threads, 0, stream>>>(a);
-    else consolidate_kernel<__nv_bfloat16, false><<<grid, threads, 0, stream>>>(a);
-  } else {
-    if (mx) consolidate_kernel<float, true><<<grid, threads, 0, stream>>>(a);
-    else consolidate_kernel<float, false><<<grid, threads, 0, stream>>>(a);
-  }
-  return cudaGetLastError();
+  void (*kern)(const ConsolidateArgs);
+  if (g.dtype == FADEMEM_BF16)
+    kern = mx ? consolidate_kernel<__nv_bfloat16, true> : consolidate_kernel<__nv_bfloat16, false>;
+  else
+    kern = mx ? consolidate_kernel<float, true> : consolidate_kernel<float, false>;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 }  // namespace fademem
