@@ -23,6 +23,7 @@ from __future__ import annotations
 import argparse
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -48,6 +49,20 @@ def _peaks():
         return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
     except Exception:
         return 6800.0, 1900.0, "fallback"
+
+
+def _profiled_traffic(profile: str, source: str):
+    """DRAM bytes per launch from a committed ncu summary, or None if the kernel
+    source changed since those counters were taken (hash recorded in the summary)."""
+    import hashlib
+    try:
+        text = open(os.path.join(ROOT, "profiles", profile)).read()
+        want = re.search(r"source_sha256_prefix:\s*([0-9a-f]+)", text).group(1)
+        traffic = int(re.search(r"traffic_bytes_per_launch:\s*(\d+)", text).group(1))
+        have = hashlib.sha256(open(os.path.join(ROOT, source), "rb").read()).hexdigest()[:len(want)]
+        return traffic if have == want else None
+    except Exception:
+        return None
 
 
 class ClockSampler:
@@ -261,11 +276,15 @@ def run_cuda(args):
         "gpu_launches": 3 * args.steps,
         "roofline": {"bound": "tensor", "kernel": "attend_tc_kernel", "achieved": round(attn_tflops, 1),
                      "peak": bf16_peak, "unit": "TFLOP/s", "frac": round(attn_tflops / bf16_peak, 4),
-                     "peak_kind": f"{peak_kind} bf16 burst", "traffic": None,
+                     "peak_kind": f"{peak_kind} bf16 burst",
+                     "traffic": _profiled_traffic("attend_tc_wan13b.md", "paper_2606_10671_gb300/csrc/attend_tc.cu"),
                      "flops_per_launch": flops, "ms_per_launch": round(attn_ms, 4)},
         "consolidate": {"bound": "hbm", "achieved": round(cons_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                         "frac": round(cons_gbs / hbm_peak, 4), "bytes_per_step": cons_bytes,
-                        "ms_per_step": round(cons_ms, 4), "plan_blocks": plan_blocks[-1]},
+                        "ms_per_step": round(cons_ms, 4), "plan_blocks": plan_blocks[-1],
+                        "note": "event time of the fademem_consolidate call: schedule kernel + consolidation kernel",
+                        "traffic": _profiled_traffic("consolidate_wan13b.md",
+                                                     "paper_2606_10671_gb300/csrc/consolidate.cu")},
         "region_ms": round(region0.elapsed_time(region1), 3),
         "clocks": clocks,
         "e2e": {"value": round(ws * LQ / (e2e_ms / 1e3), 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
