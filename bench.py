@@ -129,6 +129,26 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(x: float, device) -> float:
+    """The largest value over all ranks (the slowest replica sets the job's time).
+
+    Replicas only: the memory step has no data-path exchange (heads and layers are
+    independent and the schedule depends on frame counts alone), so each rank runs
+    its own memory and the only collective is this timing reduction.
+    """
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, step_ms: float, world: int) -> float:
+    """Units processed by all ranks per second, timed by the slowest rank (weak scaling)."""
+    return world * units_per_rank / (step_ms / 1e3)
+
+
 def _segment_inputs(seed, n_sets, device):
     """n_sets distinct (K, V, Q) segment inputs, AR(1) K/V across the sets' frames."""
     from synth import KIND_K, KIND_V, DeviceAR1, device_queries
@@ -209,12 +229,8 @@ def run_cuda(args):
     ns, nd, _ = mem.last_plan()
     plan_blocks.append(ns + nd)
     mem.device_status()
-    step_ms = (sum(t_cons) + sum(t_attn)) / args.steps
-    if ws > 1:
-        t = torch.tensor([step_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        step_ms = float(t.item())
-    value = ws * LQ / (step_ms / 1e3)
+    step_ms = max_over_ranks((sum(t_cons) + sum(t_attn)) / args.steps, dev)
+    value = whole_job_rate(LQ, step_ms, ws)
 
     hbm_peak, bf16_peak, peak_kind = _peaks()
     attn_ms = statistics.mean(t_attn)
@@ -248,11 +264,7 @@ def run_cuda(args):
         hO.copy_(out, non_blocking=True)
         b.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in e2e_ev)
-    if ws > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(statistics.mean(a.elapsed_time(b) for a, b in e2e_ev), dev)
     h2d = sum(x.numel() * x.element_size() for x in (hK[0], hV[0], hQ[0]))
     d2h = hO.numel() * hO.element_size()
     mem.device_status()
@@ -287,7 +299,7 @@ def run_cuda(args):
                                                      "paper_2606_10671_gb300/csrc/consolidate.cu")},
         "region_ms": round(region0.elapsed_time(region1), 3),
         "clocks": clocks,
-        "e2e": {"value": round(ws * LQ / (e2e_ms / 1e3), 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": round(whole_job_rate(LQ, e2e_ms, ws), 1), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms, 4)},
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
