@@ -159,6 +159,14 @@ FADEMEM_API fademem_status fademem_layer_memory(fademem_t h, int layer, void **K
  * raw word goes to *word when word is not NULL. */
 FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void *stream, uint32_t *word);
 
+/* Diagnostic of device-side failure detection: enqueues one thread that waits,
+ * through the same bounded mbarrier wait the kernels use, on a barrier that
+ * nothing signals.  After about 1 ms the wait gives up and records a time-out
+ * in the status word, so the next fademem_get_device_status returns
+ * FADEMEM_ERR_DEVICE_TIMEOUT; the CUDA context stays usable.  The paper has
+ * no counterpart.  Errors: INVALID_ARG, CUDA. */
+FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void *stream);
+
 /* Forget every entry (count = 0, t = 0).  Enqueued on stream. */
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
 

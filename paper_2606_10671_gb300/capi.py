@@ -33,7 +33,7 @@ FADEMEM_MAX_PENDING = 64
 # Every symbol include/fademem.h declares.
 EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fademem_consolidate", "fademem_attend",
            "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_layer_memory", "fademem_get_device_status",
-           "fademem_reset", "fademem_consolidate_noalloc", "fademem_destroy", "fademem_last_error")
+           "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc", "fademem_destroy", "fademem_last_error")
 
 
 class fademem_config(ctypes.Structure):
@@ -77,6 +77,7 @@ def load(path: str | None = None):
             "fademem_last_plan": (I, [P, P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)]),
             "fademem_layer_memory": (I, [P, I, ctypes.POINTER(P), ctypes.POINTER(P)]),
             "fademem_get_device_status": (I, [P, P, ctypes.POINTER(ctypes.c_uint32)]),
+            "fademem_selftest_wait_timeout": (I, [P, P]),
             "fademem_reset": (I, [P, P]),
             "fademem_consolidate_noalloc": (I, [P, P]),
             "fademem_destroy": (None, [P]),
@@ -159,6 +160,10 @@ def fademem_get_device_status(h: int, stream: int = 0, raise_on_error: bool = Tr
     if raise_on_error:
         check(st)
     return st, w.value
+
+
+def fademem_selftest_wait_timeout(h: int, stream: int = 0):
+    check(load().fademem_selftest_wait_timeout(ctypes.c_void_p(h), ctypes.c_void_p(stream)))
 
 
 def fademem_reset(h: int, stream: int = 0):

@@ -94,13 +94,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 // Bounded wait: false on time-out or when another role of the CTA aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          long long limit = kWaitLimitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitLimitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 
@@ -508,6 +509,27 @@ bool encode_3d(EncodeTiledFn enc, CUtensorMap* map, const void* base, uint64_t d
 }
 
 }  // namespace
+
+namespace {
+// Diagnostic: one thread waits, through the kernels' own bounded wait, on an
+// mbarrier that nothing arrives on; the wait gives up after `limit` cycles and
+// the time-out is recorded in the status word, as in any kernel of the library.
+__global__ void wait_selftest_kernel(unsigned int* status, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (!mbar_wait(b, 0, &abort_flag, limit)) atomicOr(status, kStatusTimeout);
+}
+}  // namespace
+
+cudaError_t launch_wait_selftest(unsigned int* status, long long limit_cycles, cudaStream_t stream) {
+  wait_selftest_kernel<<<1, 32, 0, stream>>>(status, limit_cycles);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, const void* Q, void* out, int Lq,
                                int Lk, float scale, unsigned int* status, cudaStream_t stream, char* err,

@@ -311,6 +311,16 @@ FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void* stream_,
   return FADEMEM_OK;
 }
 
+FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = launch_wait_selftest(&h->st->status, 2000000LL, stream);  // about 1 ms
+  if (e != cudaSuccess) return cuda_fail(e, "launching the wait self-test");
+  return FADEMEM_OK;
+}
+
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->need_init = true;

@@ -87,4 +87,8 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
                                int Lk, float scale, unsigned int* status, cudaStream_t stream,
                                char* err, size_t errlen);
 
+// Waits on an mbarrier that is never signalled, through the same bounded wait
+// the kernels use; sets kStatusTimeout after limit_cycles.
+cudaError_t launch_wait_selftest(unsigned int* status, long long limit_cycles, cudaStream_t stream);
+
 }  // namespace fademem

@@ -152,3 +152,19 @@ def test_wan13b_single_layer_full_size():
     Q = p.queries(4680, step=40)
     p.check_attend(Q, rows=rows)
     p.gpu.device_status()
+
+
+def test_device_wait_timeout_is_reported():
+    """A bounded device wait that runs out (a barrier nothing signals) is reported as
+    FADEMEM_ERR_DEVICE_TIMEOUT through the status word; the context stays usable."""
+    from paper_2606_10671_gb300 import capi
+    p = Pair(4, 2, 128, 64, dtype=torch.bfloat16, seed=8)
+    p.step(3)
+    capi.fademem_selftest_wait_timeout(p.gpu.handle, int(torch.cuda.current_stream().cuda_stream))
+    st, word = p.gpu.device_status(raise_on_error=False)
+    assert st == capi.FADEMEM_ERR_DEVICE_TIMEOUT and word & 1
+    st, word = p.gpu.device_status(raise_on_error=False)  # read-and-clear
+    assert st == capi.FADEMEM_OK and word == 0
+    p.step(3)  # the memory and the context still work
+    p.check_entries()
+    p.check_attend(p.queries(100))
