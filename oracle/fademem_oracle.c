@@ -258,3 +258,53 @@ int oracle_num_threads(void)
     return 1;
 #endif
 }
+
+/* Attention over the memory plus the current chunk's own keys and values (the
+ * paper's attention sees the cached entries and the frames of the chunk being
+ * generated, Sec. 4.1 / Sec. S4): the key set is every token of every entry,
+ * followed by the ncur tokens of Kcur/Vcur ([ncur][H][D]).  With ncur = 0 this
+ * is oracle_attend; with an empty memory it is attention over the chunk alone. */
+int oracle_attend_ext(const oracle_memory *m, int tokens, int H, int D, const double *Kcur, const double *Vcur,
+                      long long ncur, const double *Q, long long Lq, double scale, double *out)
+{
+    if ((long long)tokens * H * D != m->elems || (m->count == 0 && ncur == 0) || ncur < 0) return -1;
+    const long long Lmem = (long long)m->count * tokens;
+    const long long Lk = Lmem + ncur;
+    int failed = 0;
+#pragma omp parallel
+    {
+        double *logit = (double *)malloc((size_t)Lk * sizeof(double));
+        if (!logit) {
+#pragma omp atomic write
+            failed = 1;
+        }
+#pragma omp for collapse(2) schedule(dynamic, 4)
+        for (long long q = 0; q < Lq; ++q) {
+            for (int h = 0; h < H; ++h) {
+                if (!logit) continue;
+                const double *qv = Q + ((size_t)q * H + h) * D;
+                double mx = -INFINITY;
+                for (long long k = 0; k < Lk; ++k) {
+                    const double *kv = k < Lmem ? m->e[k / tokens].K + ((size_t)(k % tokens) * H + h) * D
+                                                : Kcur + ((size_t)(k - Lmem) * H + h) * D;
+                    double dot = 0.0;
+                    for (int d = 0; d < D; ++d) dot += qv[d] * kv[d];
+                    logit[k] = scale * dot;
+                    if (logit[k] > mx) mx = logit[k];
+                }
+                double Z = 0.0;
+                for (long long k = 0; k < Lk; ++k) { logit[k] = exp(logit[k] - mx); Z += logit[k]; }
+                double *o = out + ((size_t)q * H + h) * D;
+                for (int d = 0; d < D; ++d) o[d] = 0.0;
+                for (long long k = 0; k < Lk; ++k) {
+                    const double *vv = k < Lmem ? m->e[k / tokens].V + ((size_t)(k % tokens) * H + h) * D
+                                                : Vcur + ((size_t)(k - Lmem) * H + h) * D;
+                    const double p = logit[k] / Z;
+                    for (int d = 0; d < D; ++d) o[d] += p * vv[d];
+                }
+            }
+        }
+        free(logit);
+    }
+    return failed ? -2 : 0;
+}

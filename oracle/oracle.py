@@ -58,6 +58,8 @@ def _load():
         lib.oracle_entry_kv.argtypes = [P, ctypes.c_int, dp, dp]
         lib.oracle_attend.argtypes = [P, ctypes.c_int, ctypes.c_int, ctypes.c_int, dp, ctypes.c_longlong,
                                       ctypes.c_double, dp]
+        lib.oracle_attend_ext.argtypes = [P, ctypes.c_int, ctypes.c_int, ctypes.c_int, dp, dp, ctypes.c_longlong, dp,
+                                          ctypes.c_longlong, ctypes.c_double, dp]
         lib.oracle_num_threads.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -149,4 +151,19 @@ class OracleMemory:
                                      _dptr(out))
         if rc != 0:
             raise ValueError(f"oracle_attend failed ({rc})")
+        return out
+
+    def attend_ext(self, Q, Kcur, Vcur, tokens: int, heads: int, dim: int, scale: float | None = None) -> np.ndarray:
+        """Attention over every cached token followed by the current chunk's tokens
+        (Kcur, Vcur: [ncur][heads][dim], ncur may be 0)."""
+        Q = np.ascontiguousarray(Q, dtype=np.float64).reshape(-1, heads, dim)
+        Kc = np.ascontiguousarray(Kcur, dtype=np.float64).reshape(-1, heads, dim)
+        Vc = np.ascontiguousarray(Vcur, dtype=np.float64).reshape(-1, heads, dim)
+        assert Kc.shape == Vc.shape
+        out = np.empty_like(Q)
+        sc = 1.0 / np.sqrt(dim) if scale is None else float(scale)
+        rc = self._lib.oracle_attend_ext(self._h, int(tokens), int(heads), int(dim), _dptr(Kc), _dptr(Vc), Kc.shape[0],
+                                         _dptr(Q), Q.shape[0], sc, _dptr(out))
+        if rc != 0:
+            raise ValueError(f"oracle_attend_ext failed ({rc})")
         return out

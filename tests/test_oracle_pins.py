@@ -321,3 +321,26 @@ def test_oracle_rejects_bad_arguments():
         OracleMemory(4, 0.0)
     with pytest.raises(ValueError):
         OracleMemory(4, 1.5)
+
+
+def test_attention_with_current_chunk_equals_full_attention():
+    """Memory plus current chunk (the paper's cached entries + the chunk's own frames):
+    with no merges it is full attention over every frame followed by the chunk; with an
+    empty memory it is attention over the chunk alone; with no chunk it is attend()."""
+    rng = np.random.default_rng(17)
+    N, H, D, F, C = 4, 2, 8, 5, 7
+    frames = [(rng.standard_normal((N, H, D)), rng.standard_normal((N, H, D))) for _ in range(F)]
+    Kc, Vc = rng.standard_normal((C, H, D)), rng.standard_normal((C, H, D))
+    Q = rng.standard_normal((6, H, D))
+    mem = OracleMemory(8, 0.3, elems=N * H * D)
+    empty = OracleMemory(8, 0.3, elems=N * H * D)
+    np.testing.assert_allclose(empty.attend_ext(Q, Kc, Vc, N, H, D), _numpy_attention(Q, Kc, Vc, 1 / math.sqrt(D)),
+                               rtol=1e-12, atol=1e-13)
+    for K, V in frames:
+        mem.insert(K, V)
+    Kall = np.concatenate([f[0] for f in frames] + [Kc])
+    Vall = np.concatenate([f[1] for f in frames] + [Vc])
+    np.testing.assert_allclose(mem.attend_ext(Q, Kc, Vc, N, H, D), _numpy_attention(Q, Kall, Vall, 1 / math.sqrt(D)),
+                               rtol=1e-12, atol=1e-13)
+    none = np.zeros((0, H, D))
+    np.testing.assert_array_equal(mem.attend_ext(Q, none, none, N, H, D), mem.attend(Q, N, H, D))
