@@ -131,6 +131,18 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void *stream);
  * UNSUPPORTED, CUDA. */
 FADEMEM_API fademem_status fademem_attend(fademem_t h, int layer, const void *Q, void *out, int Lq, void *stream);
 
+/* Attention over the memory and the current chunk (the paper's attention sees
+ * the cached entries plus the frames of the chunk being generated: 12 history
+ * + 3 current latent frames by default, Sec. 4.1; Sec. S4).  As
+ * fademem_attend, with the key set extended by ncur >= 0 tokens whose keys and
+ * values the caller passes: Kcur, Vcur device arrays [ncur][H][D] in the
+ * config dtype (for a chunk of F frames, ncur = F * N).  With ncur = 0 this is
+ * fademem_attend; with an empty memory the queries attend over the chunk
+ * alone.  Errors: INVALID_ARG, EMPTY (no entries and ncur = 0), PENDING,
+ * UNSUPPORTED, CUDA. */
+FADEMEM_API fademem_status fademem_attend_ext(fademem_t h, int layer, const void *Q, const void *Kcur,
+                                              const void *Vcur, int ncur, void *out, int Lq, void *stream);
+
 /* Number of entries (count = min(frames seen, M)) and frames seen so far,
  * counting consolidated frames only.  Host only. */
 FADEMEM_API fademem_status fademem_counts(fademem_t h, int *count, int64_t *frames_seen);

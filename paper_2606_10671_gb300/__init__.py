@@ -100,6 +100,23 @@ class FadeMem:
         capi.fademem_attend(self.handle, layer, Q.data_ptr(), out.data_ptr(), Lq, _stream_handle(stream))
         return out
 
+    def attend_ext(self, layer: int, Q: torch.Tensor, Kcur: torch.Tensor, Vcur: torch.Tensor,
+                   out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """Attention over the memory followed by the current chunk's tokens Kcur/Vcur [ncur, H, D]."""
+        c = self.cfg
+        per = c.heads * c.head_dim
+        for X in (Q, Kcur, Vcur):
+            if X.dtype != self.dtype or X.device.type != "cuda" or not X.is_contiguous() or X.numel() % per:
+                raise ValueError("Q, Kcur and Vcur must be contiguous CUDA tensors [tokens, H, D] of the memory's dtype")
+        if Kcur.numel() != Vcur.numel():
+            raise ValueError("Kcur and Vcur hold different numbers of tokens")
+        Lq, ncur = Q.numel() // per, Kcur.numel() // per
+        if out is None:
+            out = torch.empty((Lq, c.heads, c.head_dim), dtype=self.dtype, device=Q.device)
+        capi.fademem_attend_ext(self.handle, layer, Q.data_ptr(), Kcur.data_ptr(), Vcur.data_ptr(), ncur,
+                                out.data_ptr(), Lq, _stream_handle(stream))
+        return out
+
     def counts(self):
         return capi.fademem_counts(self.handle)
 

@@ -32,6 +32,7 @@ FADEMEM_MAX_PENDING = 64
 
 # Every symbol include/fademem.h declares.
 EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fademem_consolidate", "fademem_attend",
+           "fademem_attend_ext",
            "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_layer_memory", "fademem_get_device_status",
            "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc", "fademem_destroy", "fademem_last_error")
 
@@ -72,6 +73,7 @@ def load(path: str | None = None):
             "fademem_insert": (I, [P, I, P, P, I]),
             "fademem_consolidate": (I, [P, P]),
             "fademem_attend": (I, [P, I, P, P, I, P]),
+            "fademem_attend_ext": (I, [P, I, P, P, P, I, P, I, P]),
             "fademem_counts": (I, [P, ctypes.POINTER(I), ctypes.POINTER(I64)]),
             "fademem_get_entries": (I, [P, P, I, ctypes.POINTER(I), P, P, P, P]),
             "fademem_last_plan": (I, [P, P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)]),
@@ -120,6 +122,12 @@ def fademem_consolidate(h: int, stream: int = 0):
 def fademem_attend(h: int, layer: int, Q: int, out: int, Lq: int, stream: int = 0):
     check(load().fademem_attend(ctypes.c_void_p(h), layer, ctypes.c_void_p(Q), ctypes.c_void_p(out), Lq,
                                 ctypes.c_void_p(stream)))
+
+
+def fademem_attend_ext(h: int, layer: int, Q: int, Kcur: int, Vcur: int, ncur: int, out: int, Lq: int,
+                       stream: int = 0):
+    check(load().fademem_attend_ext(ctypes.c_void_p(h), layer, ctypes.c_void_p(Q), ctypes.c_void_p(Kcur),
+                                    ctypes.c_void_p(Vcur), ncur, ctypes.c_void_p(out), Lq, ctypes.c_void_p(stream)))
 
 
 def fademem_counts(h: int):

@@ -10,11 +10,14 @@
 namespace fademem {
 namespace {
 
+// Keys: the Lk memory tokens of head h ([Lk][D] at Kc + h * head_stride), then
+// the Lk2 current-chunk tokens ([Lk2][H][D] at Kcur).
 template <int D>
 __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict__ Kc, const float* __restrict__ Vc,
+                                                         int Lk, const float* __restrict__ Kcur,
+                                                         const float* __restrict__ Vcur, int Lk2,
                                                          const float* __restrict__ Q, float* __restrict__ out,
-                                                         int Lq, int Lk, int H, size_t head_stride,
-                                                         float scale_log2) {
+                                                         int Lq, int H, size_t head_stride, float scale_log2) {
   constexpr int P = D / 32;
   const int lane = threadIdx.x & 31;
   const long long gw = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
@@ -27,10 +30,12 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
   const float* Kh = Kc + (size_t)h * head_stride;  // keys of head h: [Lk][D], slots 0..count-1 contiguous
   const float* Vh = Vc + (size_t)h * head_stride;
   float m = -INFINITY, l = 0.f;
-  for (int k = 0; k < Lk; ++k) {
+  for (int k = 0; k < Lk + Lk2; ++k) {
+    const float* kr = k < Lk ? Kh + (size_t)k * D : Kcur + ((size_t)(k - Lk) * H + h) * D;
+    const float* vr = k < Lk ? Vh + (size_t)k * D : Vcur + ((size_t)(k - Lk) * H + h) * D;
     float dot = 0.f;
 #pragma unroll
-    for (int i = 0; i < P; ++i) dot = fmaf(qv[i], Kh[(size_t)k * D + lane + 32 * i], dot);
+    for (int i = 0; i < P; ++i) dot = fmaf(qv[i], kr[lane + 32 * i], dot);
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
     const float s = dot * scale_log2;
@@ -39,7 +44,7 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
     const float p = exp2f(s - m_new);
     l = l * c + p;
 #pragma unroll
-    for (int i = 0; i < P; ++i) o[i] = fmaf(p, Vh[(size_t)k * D + lane + 32 * i], o[i] * c);
+    for (int i = 0; i < P; ++i) o[i] = fmaf(p, vr[lane + 32 * i], o[i] * c);
     m = m_new;
   }
   float* op = out + ((size_t)q * H + h) * D;
@@ -50,8 +55,9 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
 
 }  // namespace
 
-cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, const float* Q, float* out,
-                              int Lq, int Lk, float scale, cudaStream_t stream) {
+cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
+                              const void* Vcur, int Lk2, const float* Q, float* out, int Lq, float scale,
+                              cudaStream_t stream) {
   const long long warps = (long long)Lq * g.H;
   const int threads = 256;
   const long long blocks = (warps * 32 + threads - 1) / threads;
@@ -59,10 +65,12 @@ cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc,
   const size_t head_stride = (size_t)g.M * g.N * g.D;
   if (g.D == 128)
     attend_f32_kernel<128><<<(unsigned)blocks, threads, 0, stream>>>(
-        (const float*)Kc, (const float*)Vc, Q, out, Lq, Lk, g.H, head_stride, scale_log2);
+        (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
+        head_stride, scale_log2);
   else
     attend_f32_kernel<64><<<(unsigned)blocks, threads, 0, stream>>>(
-        (const float*)Kc, (const float*)Vc, Q, out, Lq, Lk, g.H, head_stride, scale_log2);
+        (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
+        head_stride, scale_log2);
   return cudaGetLastError();
 }
 

@@ -61,10 +61,12 @@ enum { BAR_Q = 0, BAR_KFULL = 1, BAR_KEMPTY = 4, BAR_VFULL = 7, BAR_VEMPTY = 9, 
 
 struct AttnParams {
   CUtensorMap tmQ;   // [Lq][H][D]  dims (D, H, Lq), box (64, 1, 128)
-  CUtensorMap tmK;   // [H][Lk][D]  dims (D, Lk, H), box (64, 128, 1)
+  CUtensorMap tmK;   // memory keys [H][Lk][D]  dims (D, Lk, H), box (64, 128, 1)
   CUtensorMap tmV;
+  CUtensorMap tmK2;  // current-chunk keys [Lk2][H][D]  dims (D, H, Lk2), box (64, 1, 128)
+  CUtensorMap tmV2;
   __nv_bfloat16* out;
-  int Lq, Lk, H;
+  int Lq, Lk, Lk2, H;
   float scale_log2;
   unsigned int* status;
 };
@@ -211,7 +213,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q0 = blockIdx.x * kBM;
   const int h = blockIdx.y;
-  const int n_tiles = (p.Lk + kBN - 1) / kBN;
+  // Key tiles 0..n1-1 come from the memory, n1..n1+n2-1 from the current chunk.
+  const int n1 = (p.Lk + kBN - 1) / kBN;
+  const int n_tiles = n1 + (p.Lk2 + kBN - 1) / kBN;
 
   if (threadIdx.x == 0) {
     s_abort = 0;
@@ -242,6 +246,10 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmQ)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmK)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmV)) : "memory");
+    if (p.Lk2 > 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmK2)) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&p.tmV2)) : "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
@@ -271,8 +279,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         }
         const uint32_t sK = sbase + kOffK + s * kTileBytes;
         mbar_expect_tx(bar(BAR_KFULL + s), kTileBytes);
-        tma_load_3d(sK, &p.tmK, bar(BAR_KFULL + s), 0, j * kBN, h);
-        tma_load_3d(sK + kHalfBytes, &p.tmK, bar(BAR_KFULL + s), 64, j * kBN, h);
+        if (j < n1) {
+          tma_load_3d(sK, &p.tmK, bar(BAR_KFULL + s), 0, j * kBN, h);
+          tma_load_3d(sK + kHalfBytes, &p.tmK, bar(BAR_KFULL + s), 64, j * kBN, h);
+        } else {
+          tma_load_3d(sK, &p.tmK2, bar(BAR_KFULL + s), 0, h, (j - n1) * kBN);
+          tma_load_3d(sK + kHalfBytes, &p.tmK2, bar(BAR_KFULL + s), 64, h, (j - n1) * kBN);
+        }
       }
     }
   } else if (warp == kWarpTmaV) {
@@ -286,8 +299,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         }
         const uint32_t sV = sbase + kOffV + s * kTileBytes;
         mbar_expect_tx(bar(BAR_VFULL + s), kTileBytes);
-        tma_load_3d(sV, &p.tmV, bar(BAR_VFULL + s), 0, j * kBN, h);
-        tma_load_3d(sV + kHalfBytes, &p.tmV, bar(BAR_VFULL + s), 64, j * kBN, h);
+        if (j < n1) {
+          tma_load_3d(sV, &p.tmV, bar(BAR_VFULL + s), 0, j * kBN, h);
+          tma_load_3d(sV + kHalfBytes, &p.tmV, bar(BAR_VFULL + s), 64, j * kBN, h);
+        } else {
+          tma_load_3d(sV, &p.tmV2, bar(BAR_VFULL + s), 0, h, (j - n1) * kBN);
+          tma_load_3d(sV + kHalfBytes, &p.tmV2, bar(BAR_VFULL + s), 64, h, (j - n1) * kBN);
+        }
       }
     }
   } else if (warp == kWarpMma) {
@@ -370,8 +388,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
           sv[96 + i] = __uint_as_float(r3[i]);
         }
       }
-      if (j == n_tiles - 1) {
-        const int valid = p.Lk - j * kBN;
+      const int valid = j < n1 ? p.Lk - j * kBN : p.Lk2 - (j - n1) * kBN;  // keys of this tile
+      if (valid < kBN) {  // the last tile of either source is ragged
 #pragma unroll
         for (int c = 0; c < kBN; ++c)
           if (c >= valid) sv[c] = -INFINITY;
@@ -531,9 +549,9 @@ cudaError_t launch_wait_selftest(unsigned int* status, long long limit_cycles, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, const void* Q, void* out, int Lq,
-                               int Lk, float scale, unsigned int* status, cudaStream_t stream, char* err,
-                               size_t errlen) {
+cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
+                               const void* Vcur, int Lk2, const void* Q, void* out, int Lq, float scale,
+                               unsigned int* status, cudaStream_t stream, char* err, size_t errlen) {
   if (g.D != kHD) {
     snprintf(err, errlen, "bf16 attention supports head_dim 128 only (got %d)", g.D);
     return cudaErrorNotSupported;
@@ -551,15 +569,23 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
   }
   AttnParams prm;
   const uint64_t row = (uint64_t)kHD * 2;
+  // An absent source (Lk == 0 or Lk2 == 0) gets a valid one-row map that no tile reads.
+  const void* k1 = Lk > 0 ? Kc : Q;
+  const void* v1 = Lk > 0 ? Vc : Q;
+  const void* k2 = Lk2 > 0 ? Kcur : Q;
+  const void* v2 = Lk2 > 0 ? Vcur : Q;
   if (!encode_3d(enc, &prm.tmQ, Q, kHD, g.H, Lq, row, row * g.H, 64, 1, kBM) ||
-      !encode_3d(enc, &prm.tmK, Kc, kHD, Lk, g.H, row, row * g.M * g.N, 64, kBN, 1) ||
-      !encode_3d(enc, &prm.tmV, Vc, kHD, Lk, g.H, row, row * g.M * g.N, 64, kBN, 1)) {
-    snprintf(err, errlen, "cuTensorMapEncodeTiled rejected a tensor map (Lq=%d Lk=%d)", Lq, Lk);
+      !encode_3d(enc, &prm.tmK, k1, kHD, Lk > 0 ? Lk : 1, g.H, row, row * g.M * g.N, 64, kBN, 1) ||
+      !encode_3d(enc, &prm.tmV, v1, kHD, Lk > 0 ? Lk : 1, g.H, row, row * g.M * g.N, 64, kBN, 1) ||
+      !encode_3d(enc, &prm.tmK2, k2, kHD, g.H, Lk2 > 0 ? Lk2 : 1, row, row * g.H, 64, 1, kBN) ||
+      !encode_3d(enc, &prm.tmV2, v2, kHD, g.H, Lk2 > 0 ? Lk2 : 1, row, row * g.H, 64, 1, kBN)) {
+    snprintf(err, errlen, "cuTensorMapEncodeTiled rejected a tensor map (Lq=%d Lk=%d Lk2=%d)", Lq, Lk, Lk2);
     return cudaErrorInvalidValue;
   }
   prm.out = reinterpret_cast<__nv_bfloat16*>(out);
   prm.Lq = Lq;
   prm.Lk = Lk;
+  prm.Lk2 = Lk2;
   prm.H = g.H;
   prm.scale_log2 = scale * 1.4426950408889634f;
   prm.status = status;

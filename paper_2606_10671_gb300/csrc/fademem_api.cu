@@ -206,32 +206,47 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   return FADEMEM_OK;
 }
 
-FADEMEM_API fademem_status fademem_attend(fademem_t h, int layer, const void* Q, void* out, int Lq, void* stream_) {
+static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const void* Kcur, const void* Vcur,
+                                  int ncur, void* out, int Lq, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
   if (!Q || !out) return fail(FADEMEM_ERR_INVALID_ARG, "Q or out is NULL");
   if (!aligned16(Q) || !aligned16(out)) return fail(FADEMEM_ERR_INVALID_ARG, "Q and out must be 16-byte aligned");
   if (Lq < 1 || Lq > (1 << 24)) return fail(FADEMEM_ERR_INVALID_ARG, "Lq must be in [1, 2^24] (got %d)", Lq);
+  if (ncur < 0 || ncur > (1 << 24)) return fail(FADEMEM_ERR_INVALID_ARG, "ncur must be in [0, 2^24] (got %d)", ncur);
+  if (ncur > 0 && (!Kcur || !Vcur)) return fail(FADEMEM_ERR_INVALID_ARG, "Kcur or Vcur is NULL");
+  if (ncur > 0 && (!aligned16(Kcur) || !aligned16(Vcur)))
+    return fail(FADEMEM_ERR_INVALID_ARG, "Kcur and Vcur must be 16-byte aligned");
   for (int l = 0; l < h->g.L; ++l)
     if (h->pending_frames[l] != 0)
       return fail(FADEMEM_ERR_PENDING, "frames inserted on layer %d await fademem_consolidate", l);
-  if (h->count == 0) return fail(FADEMEM_ERR_EMPTY, "the memory holds no entries");
+  if (h->count == 0 && ncur == 0) return fail(FADEMEM_ERR_EMPTY, "the memory holds no entries");
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   const int Lk = h->count * h->g.N;
   const char* Kc = h->cache + (size_t)layer * h->g.layer_bytes;
   const char* Vc = Kc + h->g.kv_elems * h->g.elem;
   cudaError_t e;
   if (h->g.dtype == FADEMEM_F32) {
-    e = launch_attend_f32(h->g, Kc, Vc, reinterpret_cast<const float*>(Q), reinterpret_cast<float*>(out), Lq, Lk,
-                          h->cfg.scale, stream);
+    e = launch_attend_f32(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, reinterpret_cast<const float*>(Q),
+                          reinterpret_cast<float*>(out), Lq, h->cfg.scale, stream);
   } else {
     char msg[256] = "";
-    e = launch_attend_bf16(h->g, Kc, Vc, Q, out, Lq, Lk, h->cfg.scale, &h->st->status, stream, msg, sizeof(msg));
+    e = launch_attend_bf16(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, Q, out, Lq, h->cfg.scale, &h->st->status, stream, msg,
+                           sizeof(msg));
     if (e == cudaErrorNotSupported) return fail(FADEMEM_ERR_UNSUPPORTED, "%s", msg);
     if (e == cudaErrorInvalidValue && msg[0]) return fail(FADEMEM_ERR_INVALID_ARG, "%s", msg);
   }
   if (e != cudaSuccess) return cuda_fail(e, "launching the attention kernel");
   return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_attend(fademem_t h, int layer, const void* Q, void* out, int Lq, void* stream_) {
+  return attend_impl(h, layer, Q, nullptr, nullptr, 0, out, Lq, stream_);
+}
+
+FADEMEM_API fademem_status fademem_attend_ext(fademem_t h, int layer, const void* Q, const void* Kcur,
+                                              const void* Vcur, int ncur, void* out, int Lq, void* stream_) {
+  return attend_impl(h, layer, Q, Kcur, Vcur, ncur, out, Lq, stream_);
 }
 
 FADEMEM_API fademem_status fademem_counts(fademem_t h, int* count, int64_t* frames_seen) {

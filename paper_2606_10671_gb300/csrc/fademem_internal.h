@@ -80,12 +80,15 @@ cudaError_t launch_schedule(DevState* st, int frames, int M, double beta, int an
                             cudaStream_t stream);
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
                                int frames, int op, cudaStream_t stream);
-cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, const float* Q, float* out,
-                              int Lq, int Lk, float scale, cudaStream_t stream);
+// Attention over Lk memory keys (Kc/Vc: one layer's [H][M][N][D] memory) followed
+// by Lk2 current-chunk keys (Kcur/Vcur: [Lk2][H][D]); either count may be 0.
+cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
+                              const void* Vcur, int Lk2, const float* Q, float* out, int Lq, float scale,
+                              cudaStream_t stream);
 // Returns cudaErrorNotSupported if the shape is outside the tensor-core path.
-cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, const void* Q, void* out, int Lq,
-                               int Lk, float scale, unsigned int* status, cudaStream_t stream,
-                               char* err, size_t errlen);
+cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
+                               const void* Vcur, int Lk2, const void* Q, void* out, int Lq, float scale,
+                               unsigned int* status, cudaStream_t stream, char* err, size_t errlen);
 
 // Waits on an mbarrier that is never signalled, through the same bounded wait
 // the kernels use; sets kStatusTimeout after limit_cycles.

@@ -174,6 +174,25 @@ class Pair:
         q = host_queries((Lq, self.H, self.D), self.seed, layer, step)
         return torch.from_numpy(q).to(self.dtype).cuda()
 
+    def chunk(self, ncur, step=0, layer=0):
+        """Keys and values of a current chunk [ncur, H, D] (its own stream, N(0,1))."""
+        g = np.random.default_rng([self.seed, 77, layer, step])
+        K = g.standard_normal((ncur, self.H, self.D), dtype=np.float32)
+        V = g.standard_normal((ncur, self.H, self.D), dtype=np.float32)
+        return torch.from_numpy(K).to(self.dtype).cuda(), torch.from_numpy(V).to(self.dtype).cuda()
+
+    def check_attend_ext(self, Q: torch.Tensor, Kcur: torch.Tensor, Vcur: torch.Tensor, layer=0, rows=None):
+        out = self.gpu.attend_ext(layer, Q, Kcur, Vcur)
+        torch.cuda.synchronize()
+        if rows is not None:
+            idx = torch.as_tensor(np.asarray(rows), device=Q.device)
+            Q, out = Q[idx], out[idx]
+        Qt = Q.double().cpu().numpy()[:, self.tracked, :]
+        Kc = Kcur.double().cpu().numpy()[:, self.tracked, :]
+        Vc = Vcur.double().cpu().numpy()[:, self.tracked, :]
+        ref = self.ora[layer].attend_ext(Qt, Kc, Vc, self.N, len(self.tracked), self.D)
+        return assert_close(out.double().cpu().numpy()[:, self.tracked, :], ref, self.dtype, "attention + chunk")
+
     def check_attend(self, Q: torch.Tensor, layer=0, rows=None):
         out = self.gpu.attend(layer, Q)
         torch.cuda.synchronize()

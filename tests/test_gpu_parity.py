@@ -168,3 +168,27 @@ def test_device_wait_timeout_is_reported():
     p.step(3)  # the memory and the context still work
     p.check_entries()
     p.check_attend(p.queries(100))
+
+
+@pytest.mark.parametrize("dtype,D,N,M,Lq", [(torch.float32, 64, 64, 8, 192), (torch.bfloat16, 128, 100, 5, 300)])
+def test_attend_with_current_chunk(dtype, D, N, M, Lq):
+    """15-slot attention: memory entries plus the current chunk's 3 frames (ncur = 3N).
+    Segment 0 attends over its own chunk alone (empty memory); bf16 keys are ragged in
+    both sources (memory 5x100 = 3 tiles + 116, chunk 300 = 2 tiles + 44)."""
+    p = Pair(M, 2, D, N, beta=0.3, dtype=dtype, seed=9)
+    for seg in range(8):
+        Kc, Vc = p.chunk(3 * N, step=seg)
+        p.check_attend_ext(p.queries(Lq, step=seg), Kc, Vc)
+        p.step(3)
+    Kc, Vc = p.chunk(0, step=99)
+    p.check_attend_ext(p.queries(Lq, step=99), Kc, Vc)  # ncur = 0: plain attention
+
+
+def test_attend_with_current_chunk_full_size():
+    """Wan-1.3B shape: 21 entries (32,760 keys/head) + the 3-frame chunk (4,680 keys), sampled rows."""
+    p = Pair(21, 12, 128, 1560, beta=0.3, dtype=torch.bfloat16, seed=10, tracked_heads=[3, 9], device_gen=True)
+    for seg in range(9):
+        p.step(3)
+    Kc, Vc = p.chunk(4680, step=1)
+    rows = np.array([0, 5, 1234, 4095, 4679])
+    p.check_attend_ext(p.queries(4680, step=9), Kc, Vc, rows=rows)
