@@ -6,7 +6,7 @@
 // One CTA computes one 128-query tile of one head, 352 threads:
 //   warp 8      TMA producer of Q (once) and of K tiles of 128 keys into a
 //               3-stage ring (128-byte swizzle, zero fill past the last key)
-//   warp 10     TMA producer of V tiles into a 2-stage ring, so a slow V slot
+//   warp 10     TMA producer of V tiles into a 3-stage ring, so a slow V slot
 //               never holds back the next K tile
 //   warp 9      allocates 512 TMEM columns and issues tcgen05.mma
 //   warps 0-7   two softmax groups of four warps; group g takes the key tiles
@@ -40,15 +40,17 @@ constexpr int kWarpMma = 9;
 constexpr int kWarpTmaV = 10;  // V producer
 constexpr int kThreads = 352;
 constexpr int kKStages = 3;
-constexpr int kVStages = 2;
+constexpr int kVStages = 3;
 constexpr uint32_t kHalfBytes = kBM * 64 * 2;   // 128 rows x 64 bf16 (one swizzle-128B panel)
 constexpr uint32_t kTileBytes = 2 * kHalfBytes; // 128 rows x 128 bf16
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = kOffQ + kTileBytes;
 constexpr uint32_t kOffV = kOffK + kKStages * kTileBytes;
 constexpr uint32_t kOffBar = kOffV + kVStages * kTileBytes;
-constexpr uint32_t kOffML = kOffBar + 256;           // per-row (m, l) of both groups
-constexpr uint32_t kSmemBytes = kOffML + 4 * kBM * 4 + 1024;  // + alignment slack
+// Per-row (m, l) of both groups for the epilogue: reuses K stage 0, which no
+// MMA reads any more once the final drain has completed.
+constexpr uint32_t kOffML = kOffK;
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;  // + alignment slack
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: S_0 [0,128), S_1 [128,256) fp32 (P_g overwrites the first 64
 // columns of S_g as bf16 pairs); O_0 [256,384), O_1 [384,512) fp32.
@@ -56,8 +58,8 @@ constexpr uint32_t kColO = 256;
 constexpr long long kWaitLimitCycles = 4000000000LL;  // ~2 s at 2 GHz
 
 // Barrier indices (8 bytes each at kOffBar).
-enum { BAR_Q = 0, BAR_KFULL = 1, BAR_KEMPTY = 4, BAR_VFULL = 7, BAR_VEMPTY = 9, BAR_SFULL = 11, BAR_PFULL = 13,
-       BAR_FINAL = 15, BAR_COUNT = 16 };
+enum { BAR_Q = 0, BAR_KFULL = 1, BAR_KEMPTY = 4, BAR_VFULL = 7, BAR_VEMPTY = 10, BAR_SFULL = 13, BAR_PFULL = 15,
+       BAR_FINAL = 17, BAR_COUNT = 18 };
 
 struct AttnParams {
   CUtensorMap tmQ;   // [Lq][H][D]  dims (D, H, Lq), box (64, 1, 128)
@@ -195,9 +197,56 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// Packed two-lane fp32 arithmetic (one instruction for two values): the
+// softmax is bound by instruction issue, so pairs halve its FFMA/FADD count.
+__device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, float b0, float b1, float c0,
+                                      float c1) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+__device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&b);
+}
+
+__device__ __forceinline__ uint32_t barat(uint32_t bar0, int i) { return bar0 + 8u * (uint32_t)i; }
+
+__device__ __noinline__ void record_timeout(volatile int* abort_flag, unsigned int* status) {
+  *abort_flag = 1;
+  atomicOr(status, kStatusTimeout);
+}
+
+// The 8 MMAs (K = 128 in steps of 16) of S = Q K^T for one key tile, issued
+// back to back: every operand is a by-value register and the descriptors only
+// advance by constants, so nothing between two tcgen05.mma stalls the issuer.
+__device__ __forceinline__ void issue_qk8(uint32_t tS, uint64_t dQ, uint64_t dK, uint32_t idesc) {
+#pragma unroll
+  for (int kk = 0; kk < kHD / 16; ++kk) {
+    const uint64_t off = (uint64_t)(((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4);
+    umma_bf16(tS, dQ + off, dK + off, idesc, kk > 0 ? 1u : 0u);
+  }
+}
+// The 8 MMAs of O += P V for one key tile (P in TMEM, 16 keys = 8 columns per step).
+__device__ __forceinline__ void issue_pv8(uint32_t tO, uint32_t tP, uint64_t dV, uint32_t idesc, uint32_t acc0) {
+#pragma unroll
+  for (int kk = 0; kk < kBN / 16; ++kk)
+    umma_bf16_ts(tO, tP + kk * 8, dV + (uint64_t)(kk * (2048 >> 4)), idesc, kk > 0 ? 1u : acc0);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_constant__ AttnParams p) {
@@ -205,7 +254,6 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = sbase + kOffBar;
-  auto bar = [&](int i) { return bar0 + 8u * i; };
   float* s_ml = reinterpret_cast<float*>(smem + kOffML);  // [2 groups][2 (m, l)][128 rows]
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
@@ -219,20 +267,20 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
 
   if (threadIdx.x == 0) {
     s_abort = 0;
-    mbar_init(bar(BAR_Q), 1);
+    mbar_init(barat(bar0, BAR_Q), 1);
     for (int s = 0; s < kKStages; ++s) {
-      mbar_init(bar(BAR_KFULL + s), 1);
-      mbar_init(bar(BAR_KEMPTY + s), 1);
+      mbar_init(barat(bar0, BAR_KFULL + s), 1);
+      mbar_init(barat(bar0, BAR_KEMPTY + s), 1);
     }
     for (int s = 0; s < kVStages; ++s) {
-      mbar_init(bar(BAR_VFULL + s), 1);
-      mbar_init(bar(BAR_VEMPTY + s), 1);
+      mbar_init(barat(bar0, BAR_VFULL + s), 1);
+      mbar_init(barat(bar0, BAR_VEMPTY + s), 1);
     }
     for (int g = 0; g < 2; ++g) {
-      mbar_init(bar(BAR_SFULL + g), 1);
-      mbar_init(bar(BAR_PFULL + g), 128);
+      mbar_init(barat(bar0, BAR_SFULL + g), 1);
+      mbar_init(barat(bar0, BAR_PFULL + g), 128);
     }
-    mbar_init(bar(BAR_FINAL), 1);
+    mbar_init(barat(bar0, BAR_FINAL), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -259,52 +307,50 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const uint32_t tmem = s_tmem;
   volatile int* abort_flag = &s_abort;
-  auto fail = [&]() {
-    *abort_flag = 1;
-    atomicOr(p.status, kStatusTimeout);
-  };
 
   if (warp == kWarpTma) {
     // ---------------- TMA producer of Q (once) and K_j into stage j%3 ----------------
     if (lane == 0) {
       const uint32_t sQ = sbase + kOffQ;
-      mbar_expect_tx(bar(BAR_Q), kTileBytes);
-      tma_load_3d(sQ, &p.tmQ, bar(BAR_Q), 0, h, q0);
-      tma_load_3d(sQ + kHalfBytes, &p.tmQ, bar(BAR_Q), 64, h, q0);
+      mbar_expect_tx(barat(bar0, BAR_Q), kTileBytes);
+      tma_load_3d(sQ, &p.tmQ, barat(bar0, BAR_Q), 0, h, q0);
+      tma_load_3d(sQ + kHalfBytes, &p.tmQ, barat(bar0, BAR_Q), 64, h, q0);
       for (int j = 0; j < n_tiles; ++j) {
         const int s = j % kKStages;
-        if (j >= kKStages && !mbar_wait(bar(BAR_KEMPTY + s), ((j / kKStages) & 1) ^ 1, abort_flag)) {
-          fail();
+        const uint32_t full = barat(bar0, BAR_KFULL + s);
+        if (j >= kKStages && !mbar_wait(barat(bar0, BAR_KEMPTY + s), ((j / kKStages) & 1) ^ 1, abort_flag)) {
+          record_timeout(abort_flag, p.status);
           break;
         }
         const uint32_t sK = sbase + kOffK + s * kTileBytes;
-        mbar_expect_tx(bar(BAR_KFULL + s), kTileBytes);
+        mbar_expect_tx(full, kTileBytes);
         if (j < n1) {
-          tma_load_3d(sK, &p.tmK, bar(BAR_KFULL + s), 0, j * kBN, h);
-          tma_load_3d(sK + kHalfBytes, &p.tmK, bar(BAR_KFULL + s), 64, j * kBN, h);
+          tma_load_3d(sK, &p.tmK, full, 0, j * kBN, h);
+          tma_load_3d(sK + kHalfBytes, &p.tmK, full, 64, j * kBN, h);
         } else {
-          tma_load_3d(sK, &p.tmK2, bar(BAR_KFULL + s), 0, h, (j - n1) * kBN);
-          tma_load_3d(sK + kHalfBytes, &p.tmK2, bar(BAR_KFULL + s), 64, h, (j - n1) * kBN);
+          tma_load_3d(sK, &p.tmK2, full, 0, h, (j - n1) * kBN);
+          tma_load_3d(sK + kHalfBytes, &p.tmK2, full, 64, h, (j - n1) * kBN);
         }
       }
     }
   } else if (warp == kWarpTmaV) {
-    // ---------------- TMA producer of V_j into stage j%2 (independent of the K ring) ----------------
+    // ---------------- TMA producer of V_j into stage j%3 (independent of the K ring) ----------------
     if (lane == 0) {
       for (int j = 0; j < n_tiles; ++j) {
         const int s = j % kVStages;
-        if (j >= kVStages && !mbar_wait(bar(BAR_VEMPTY + s), ((j / kVStages) & 1) ^ 1, abort_flag)) {
-          fail();
+        const uint32_t full = barat(bar0, BAR_VFULL + s);
+        if (j >= kVStages && !mbar_wait(barat(bar0, BAR_VEMPTY + s), ((j / kVStages) & 1) ^ 1, abort_flag)) {
+          record_timeout(abort_flag, p.status);
           break;
         }
         const uint32_t sV = sbase + kOffV + s * kTileBytes;
-        mbar_expect_tx(bar(BAR_VFULL + s), kTileBytes);
+        mbar_expect_tx(full, kTileBytes);
         if (j < n1) {
-          tma_load_3d(sV, &p.tmV, bar(BAR_VFULL + s), 0, j * kBN, h);
-          tma_load_3d(sV + kHalfBytes, &p.tmV, bar(BAR_VFULL + s), 64, j * kBN, h);
+          tma_load_3d(sV, &p.tmV, full, 0, j * kBN, h);
+          tma_load_3d(sV + kHalfBytes, &p.tmV, full, 64, j * kBN, h);
         } else {
-          tma_load_3d(sV, &p.tmV2, bar(BAR_VFULL + s), 0, h, (j - n1) * kBN);
-          tma_load_3d(sV + kHalfBytes, &p.tmV2, bar(BAR_VFULL + s), 64, h, (j - n1) * kBN);
+          tma_load_3d(sV, &p.tmV2, full, 0, h, (j - n1) * kBN);
+          tma_load_3d(sV + kHalfBytes, &p.tmV2, full, 64, h, (j - n1) * kBN);
         }
       }
     }
@@ -314,51 +360,47 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
     // writes P_j over the first 64 columns of that buffer, and P_j V_j goes to the
     // group's own accumulator O_{j%2}.  The tensor pipe runs tcgen05.mma in issue
     // order, so issuing S_{j+2} after P_j V_j never overwrites P_j too early.
+    // One commit per tile: a commit costs the tensor pipe about as much as an MMA,
+    // so K/V slot release is signalled by the softmax groups, not here.
     if (lane == 0) {
       constexpr uint32_t idesc_qk = make_idesc(kBM, kBN, 0);
       constexpr uint32_t idesc_pv = make_idesc(kBM, kHD, 1);
-      // Descriptors are built once per operand buffer and advanced along K by adding
-      // (byte offset >> 4) to the start-address field: the issuing thread must not
-      // spend a dependent integer chain per MMA, or issue (not the tensor pipe) limits.
       const uint64_t dQ = sw128_desc(sbase + kOffQ, 16, 1024);
-      auto issue_qk = [&](int j) -> bool {
+      const uint64_t dK0 = sw128_desc(sbase + kOffK, 16, 1024);
+      const uint64_t dV0 = sw128_desc(sbase + kOffV, kHalfBytes, 1024);
+      constexpr uint64_t kStageStep = kTileBytes >> 4;  // descriptor advance per 32 KB stage
+      bool ok = mbar_wait(barat(bar0, BAR_Q), 0, abort_flag);
+      for (int j = 0; ok && j < 2 && j < n_tiles; ++j) {
         const int s = j % kKStages;
-        if (!mbar_wait(bar(BAR_KFULL + s), (j / kKStages) & 1, abort_flag)) return false;
+        if (!mbar_wait(barat(bar0, BAR_KFULL + s), (j / kKStages) & 1, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        const uint64_t dK = sw128_desc(sbase + kOffK + s * kTileBytes, 16, 1024);
-        const uint32_t tS = tmem + (j & 1) * kBN;
-#pragma unroll
-        for (int kk = 0; kk < kHD / 16; ++kk) {
-          const uint64_t off = ((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4;
-          umma_bf16(tS, dQ + off, dK + off, idesc_qk, kk > 0);
-        }
-        umma_commit(bar(BAR_SFULL + (j & 1)));
-        umma_commit(bar(BAR_KEMPTY + s));
-        return true;
-      };
-      bool ok = mbar_wait(bar(BAR_Q), 0, abort_flag);
-      if (!ok) fail();
-      tc_fence_after();
-      for (int j = 0; ok && j < 2 && j < n_tiles; ++j)
-        if (!issue_qk(j)) { fail(); ok = false; }
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const int g = j & 1, s = j % kVStages;
-        if (!mbar_wait(bar(BAR_PFULL + g), (j >> 1) & 1, abort_flag)) { fail(); break; }
-        if (!mbar_wait(bar(BAR_VFULL + s), (j / kVStages) & 1, abort_flag)) { fail(); break; }
-        tc_fence_after();
-        const uint64_t dV = sw128_desc(sbase + kOffV + s * kTileBytes, kHalfBytes, 1024);
-        const uint32_t tP = tmem + g * kBN;
-        const uint32_t tO = tmem + kColO + g * kHD;
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          umma_bf16_ts(tO, tP + kk * 8, dV + (uint64_t)(kk * (2048 >> 4)), idesc_pv, (j >= 2 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(bar(BAR_VEMPTY + s));
-        if (j + 2 < n_tiles && !issue_qk(j + 2)) { fail(); break; }
+        issue_qk8(tmem + (j & 1) * kBN, dQ, dK0 + s * kStageStep, idesc_qk);
+        umma_commit(barat(bar0, BAR_SFULL + (j & 1)));
       }
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int g = j & 1, sv = j % kVStages;
+        if (!mbar_wait(barat(bar0, BAR_PFULL + g), (j >> 1) & 1, abort_flag) ||
+            !mbar_wait(barat(bar0, BAR_VFULL + sv), (j / kVStages) & 1, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        issue_pv8(tmem + kColO + g * kHD, tmem + g * kBN, dV0 + sv * kStageStep, idesc_pv, j >= 2 ? 1u : 0u);
+        const int jn = j + 2;
+        if (jn < n_tiles) {
+          const int sk = jn % kKStages;
+          if (!mbar_wait(barat(bar0, BAR_KFULL + sk), (jn / kKStages) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          issue_qk8(tmem + g * kBN, dQ, dK0 + sk * kStageStep, idesc_qk);
+          // Completes with P_j V_j and S_{j+2}: the group's next S, and (through it)
+          // the release of V slot j%3 and K slot (j+2)%3.
+          umma_commit(barat(bar0, BAR_SFULL + g));
+        }
+      }
+      if (!ok && !*abort_flag) record_timeout(abort_flag, p.status);
       // Drain: every MMA issued above has completed once this barrier flips.
-      umma_commit(bar(BAR_FINAL));
-      if (!mbar_wait(bar(BAR_FINAL), 0, abort_flag) && !*abort_flag) fail();
+      umma_commit(barat(bar0, BAR_FINAL));
+      if (!mbar_wait(barat(bar0, BAR_FINAL), 0, abort_flag) && !*abort_flag) record_timeout(abort_flag, p.status);
     }
   } else {
     // ---------------- softmax groups 0/1 (warps 0-3 / 4-7), one query row per thread ----------------
@@ -370,7 +412,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
     for (int j = grp; j < n_tiles; j += 2) {
-      if (!mbar_wait(bar(BAR_SFULL + grp), (j >> 1) & 1, abort_flag)) { fail(); ok = false; break; }
+      if (!mbar_wait(barat(bar0, BAR_SFULL + grp), (j >> 1) & 1, abort_flag)) { record_timeout(abort_flag, p.status); ok = false; break; }
+      if ((threadIdx.x & 127) == 0) {
+        // S_j complete means Q K_j^T and (issued before it) P_{j-2} V_{j-2} are done:
+        // K slot j%3 and V slot (j-2)%3 may be refilled.
+        mbar_arrive(barat(bar0, BAR_KEMPTY + j % kKStages));
+        if (j >= 2) mbar_arrive(barat(bar0, BAR_VEMPTY + (j - 2) % kVStages));
+      }
       tc_fence_after();
       float sv[kBN];
       {
@@ -396,13 +444,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
       }
       float mx[8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) mx[k] = sv[k];
+      for (int k = 0; k < 8; ++k) mx[k] = fmaxf(sv[2 * k], sv[2 * k + 1]);
 #pragma unroll
-      for (int c = 8; c < kBN; c += 8)
+      for (int c = 16; c < kBN; c += 16)
 #pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = fmaxf(mx[k], sv[c + k]);
-      const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                             fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * p.scale_log2;
+        for (int k = 0; k < 8; ++k) mx[k] = fmax3(mx[k], sv[c + 2 * k], sv[c + 2 * k + 1]);
+      const float mt = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) *
+                       p.scale_log2;
       // Lazy reference maximum: move it only when the tile exceeds it by > 8 (2^8 headroom).
       const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
       const float m_new = move ? fmaxf(mt, m_run) : m_run;
@@ -413,10 +461,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         uint32_t pk[16];
 #pragma unroll
         for (int c = 0; c < 32; c += 2) {
-          const float e0 = ex2(fmaf(sv[32 * qtr + c], p.scale_log2, -m_new));
-          const float e1 = ex2(fmaf(sv[32 * qtr + c + 1], p.scale_log2, -m_new));
-          rs0 += e0;
-          rs1 += e1;
+          float x0, x1;
+          ffma2(x0, x1, sv[32 * qtr + c], sv[32 * qtr + c + 1], p.scale_log2, p.scale_log2, -m_new, -m_new);
+          const float e0 = ex2(x0);
+          const float e1 = ex2(x1);
+          fadd2(rs0, rs1, rs0, rs1, e0, e1);
           pk[c / 2] = pack_bf16(e0, e1);
         }
         tmem_st16(tS + qtr * 16, pk);  // P over the first 64 columns of the S buffer
@@ -438,16 +487,16 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
       }
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(bar(BAR_PFULL + grp));
+      mbar_arrive(barat(bar0, BAR_PFULL + grp));
     }
     // ---------------- epilogue: combine the two groups' (O, m, l) ----------------
-    s_ml[(grp * 2 + 0) * kBM + row] = m_run;
+    const bool fin = ok && !*abort_flag && mbar_wait(barat(bar0, BAR_FINAL), 0, abort_flag);
+    if (ok && !fin) record_timeout(abort_flag, p.status);
+    s_ml[(grp * 2 + 0) * kBM + row] = m_run;  // K stage 0 is idle once every MMA has completed
     s_ml[(grp * 2 + 1) * kBM + row] = l_run;
     asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
-    if (ok && !*abort_flag) {
-      if (!mbar_wait(bar(BAR_FINAL), 0, abort_flag)) {
-        fail();
-      } else {
+    if (fin && !*abort_flag) {
+      {
         tc_fence_after();
         const float m0 = s_ml[0 * kBM + row], l0 = s_ml[1 * kBM + row];
         const float m1 = s_ml[2 * kBM + row], l1 = s_ml[3 * kBM + row];
