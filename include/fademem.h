@@ -120,6 +120,11 @@ FADEMEM_API fademem_status fademem_insert(fademem_t h, int layer, const void *K,
  * block read once, each changed slot written once).  Asynchronous on stream.
  * Storage slots: the merged entry keeps m_j's slot, the new entry takes
  * m_{j+1}'s; occupied slots are always 0..count-1.
+ * The schedule depends on the entry table alone, so the consolidation kernel
+ * of a single-pass call also schedules the next pass (assuming the same number
+ * of frames) into a second entry-table buffer of the workspace; the next call
+ * with that frame count then launches only the consolidation kernel, and any
+ * other count schedules as usual.
  * Errors: INVALID_ARG (layers with different pending frames), CUDA. */
 FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void *stream);
 
@@ -161,6 +166,16 @@ FADEMEM_API fademem_status fademem_get_entries(fademem_t h, void *stream, int ca
  * K and V per layer: the algorithmic HBM traffic of the consolidation. */
 FADEMEM_API fademem_status fademem_last_plan(fademem_t h, void *stream, int *n_src, int *n_dest, int *frames);
 
+/* Counters (synchronises stream; any out pointer may be NULL).  Kept on the
+ * device since create/reset: *blocks_moved = the sum over consolidation
+ * passes of (sources read + slots written), each block one entry's K and V
+ * of every layer, so the algorithmic HBM bytes of all passes are
+ * blocks_moved * L * 2*N*H*D*elem; *passes = consolidation passes.  Kept on
+ * the host since create (not cleared by reset): *kernel_launches = kernels
+ * this handle has launched (schedule, consolidation, attention, self-test). */
+FADEMEM_API fademem_status fademem_stats(fademem_t h, void *stream, uint64_t *blocks_moved, uint64_t *passes,
+                                        uint64_t *kernel_launches);
+
 /* Device pointers to one layer's stored K and V memory, each laid out as
  * [H][M][N][D] in the storage dtype; storage slot s of head h starts at
  * ((h * M) + s) * N * D elements.  Only slots 0..count-1 hold entries. */
@@ -187,15 +202,16 @@ FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
 
 /* fademem_consolidate without any scratch in the caller's workspace and without
  * any allocation (no cudaMalloc, cudaFree or allocating library call): the
- * per-call working state (a copy of the entry table, the merge plan and the
- * status word) lives in a file-scope device array of the library, of
+ * per-call working state (a copy of the entry table and the merge plan)
+ * lives in a file-scope device array of the library, of
  * FADEMEM_NOALLOC_SCRATCH_BYTES bytes, that every GPU which loads the library
  * holds until the process exits.  The paper has no counterpart: this serves
  * callers that may not allocate device memory once they are running, such as
  * plug-ins of a host framework that owns all device memory, or real-time loops
  * that fix their memory at start-up.  The caller still passes the memory
  * (workspace of fademem_create) and the inserted frames, as for
- * fademem_consolidate, and the results are the same.
+ * fademem_consolidate, and the results are the same.  The device status word
+ * stays in the workspace; no schedule is computed ahead.
  * The first call on each device looks up the array's device address with that
  * device current (cudaGetSymbolAddress); make that first call before any
  * stream capture.  Every call shares the one array: calls that overlap on the

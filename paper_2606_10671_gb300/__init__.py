@@ -128,6 +128,10 @@ class FadeMem:
         """(n_src, n_dest, frames) of the latest consolidation pass."""
         return capi.fademem_last_plan(self.handle, _stream_handle(stream))
 
+    def stats(self, stream=None):
+        """(blocks moved, consolidation passes) since create/reset, kernels launched since create."""
+        return capi.fademem_stats(self.handle, _stream_handle(stream))
+
     def layer_memory(self, layer: int):
         """(K, V) torch views [H, M, N, D] of one layer's stored memory (slots 0..count-1 valid)."""
         c = self.cfg

@@ -33,7 +33,8 @@ FADEMEM_MAX_PENDING = 64
 # Every symbol include/fademem.h declares.
 EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fademem_consolidate", "fademem_attend",
            "fademem_attend_ext",
-           "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_layer_memory", "fademem_get_device_status",
+           "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_stats",
+           "fademem_layer_memory", "fademem_get_device_status",
            "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc", "fademem_destroy", "fademem_last_error")
 
 
@@ -77,6 +78,8 @@ def load(path: str | None = None):
             "fademem_counts": (I, [P, ctypes.POINTER(I), ctypes.POINTER(I64)]),
             "fademem_get_entries": (I, [P, P, I, ctypes.POINTER(I), P, P, P, P]),
             "fademem_last_plan": (I, [P, P, ctypes.POINTER(I), ctypes.POINTER(I), ctypes.POINTER(I)]),
+            "fademem_stats": (I, [P, P, ctypes.POINTER(ctypes.c_uint64), ctypes.POINTER(ctypes.c_uint64),
+                                  ctypes.POINTER(ctypes.c_uint64)]),
             "fademem_layer_memory": (I, [P, I, ctypes.POINTER(P), ctypes.POINTER(P)]),
             "fademem_get_device_status": (I, [P, P, ctypes.POINTER(ctypes.c_uint32)]),
             "fademem_selftest_wait_timeout": (I, [P, P]),
@@ -154,6 +157,13 @@ def fademem_last_plan(h: int, stream: int = 0):
     check(load().fademem_last_plan(ctypes.c_void_p(h), ctypes.c_void_p(stream), ctypes.byref(ns), ctypes.byref(nd),
                                    ctypes.byref(nf)))
     return ns.value, nd.value, nf.value
+
+
+def fademem_stats(h: int, stream: int = 0):
+    b, n, k = ctypes.c_uint64(), ctypes.c_uint64(), ctypes.c_uint64()
+    check(load().fademem_stats(ctypes.c_void_p(h), ctypes.c_void_p(stream), ctypes.byref(b), ctypes.byref(n),
+                               ctypes.byref(k)))
+    return b.value, n.value, k.value
 
 
 def fademem_layer_memory(h: int, layer: int):

@@ -71,29 +71,28 @@ __device__ __forceinline__ void warp_argmin(double& v, int& i) {
 // the smallest upper bound U = min_k (g32_k + E_k) are scored again in fp64.
 // A pair outside that set has a true gap above the true minimum by more than
 // the fp64 rounding, so it cannot be the fp64 argmin either.
-__global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, int M, double beta, int anchor,
-                                                      int op, int expected_count) {
-  __shared__ SchedShared s;
-  const int lane = threadIdx.x;
-  // The consolidation kernel launched after this one may start now: it waits
-  // for this grid's completion before it reads the plan.
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  DevMeta& m = st->meta;
-  int count = m.count;
+// Reads the entry table of `in` and writes the updated table and the pass's
+// merge plan to `out` (the same state for an in-place pass, another buffer
+// for a pass scheduled ahead of its frames).  Run by one full warp.
+__device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, DevState* out, unsigned int* status,
+                                           int frames, int M, double beta, int anchor, int op, int expected_count) {
+  const int lane = threadIdx.x & 31;
+  const DevMeta& mi = in->meta;
+  int count = mi.count;
   if (count != expected_count || count < 0 || count > M) {
-    if (lane == 0) atomicOr(&st->status, kStatusCountMismatch);
-    if (lane == 0) st->plan.n_src = 0;
+    if (lane == 0) atomicOr(status, kStatusCountMismatch);
+    if (lane == 0) out->plan.n_src = 0;
     return;
   }
-  const long long t0 = m.t_next;
+  const long long t0 = mi.t_next;
   const float beta32 = (float)beta;
   for (int i = lane; i < count; i += 32) {
-    s.slot[i] = m.slot[i];
-    s.first[i] = m.first[i];
-    s.span[i] = m.span[i];
-    s.mu2[i] = __double2ll_rn(2.0 * m.mu[i]);
+    s.slot[i] = mi.slot[i];
+    s.first[i] = mi.first[i];
+    s.span[i] = mi.span[i];
+    s.mu2[i] = __double2ll_rn(2.0 * mi.mu[i]);
     s.natoms[i] = 1;
-    s.ref[i][0] = m.slot[i];  // content: the block now stored in its own slot
+    s.ref[i][0] = mi.slot[i];  // content: the block now stored in its own slot
     s.w[i][0] = 1.0f;
   }
   __syncwarp();
@@ -242,7 +241,9 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     ns += __shfl_sync(0xffffffffu, incl, 31);
   }
   __syncwarp();
-  DevPlan& p = st->plan;
+  __syncwarp();  // every lane has read `in` before `out` (possibly the same) is written
+  DevPlan& p = out->plan;
+  DevMeta& m = out->meta;
   const bool overflow = nd > kMaxDest || ns > kMaxSrc;
   if (!overflow) {
     for (int i = lane; i < count; i += 32) {
@@ -258,7 +259,7 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     }
   }
   if (lane == 0) {
-    if (overflow) { nd = 0; ns = 0; atomicOr(&st->status, kStatusPlanOverflow); }
+    if (overflow) { nd = 0; ns = 0; atomicOr(status, kStatusPlanOverflow); }
     p.n_src = ns;
     p.n_dest = nd;
     p.frames = frames;
@@ -273,6 +274,16 @@ __global__ void __launch_bounds__(32) schedule_kernel(DevState* st, int frames, 
     m.span[i] = s.span[i];
     m.mu[i] = 0.5 * (double)s.mu2[i];
   }
+}
+
+__global__ void __launch_bounds__(32) schedule_kernel(const DevState* in, DevState* out, unsigned int* status,
+                                                      int frames, int M, double beta, int anchor, int op,
+                                                      int expected_count) {
+  __shared__ SchedShared s;
+  // The consolidation kernel launched after this one may start now: it waits
+  // for this grid's completion before it reads the plan.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  schedule_pass(s, in, out, status, frames, M, beta, anchor, op, expected_count);
 }
 
 // ---- K2 ------------------------------------------------------------------
@@ -317,11 +328,22 @@ struct ConsolidateArgs {
   size_t slab_elems;      // N * D
   size_t kv_elems;        // H * M * N * D
   size_t layer_elems;     // stride between layers, in elements
+  // Lookahead: the last row of the grid (one block) schedules the next pass of
+  // la_frames units from la_in's entry table into la_out (skipped if null).
+  const DevState* la_in;
+  DevState* la_out;
+  unsigned int* status;
+  unsigned long long* totals;  // [blocks moved, passes] since the memory was created
+  int la_frames, la_expected, la_anchor, la_op;
+  double la_beta;
   PassSources srcs;
 };
 
+constexpr int kConsolidateBlocksPerSM = 3;  // resident 256-thread blocks per SM (register-limited)
+
 template <typename T, bool kMax>
-__global__ void __launch_bounds__(256) consolidate_kernel(const __grid_constant__ ConsolidateArgs a) {
+__global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kernel(
+    const __grid_constant__ ConsolidateArgs a) {
   using V = Vec<T>;
   __shared__ int s_ref[kMaxSrc], s_dest[kMaxSrc], s_dslot[kMaxDest];
   __shared__ float s_w[kMaxSrc];
@@ -329,6 +351,15 @@ __global__ void __launch_bounds__(256) consolidate_kernel(const __grid_constant_
   // Launched as a programmatic dependent of the schedule kernel: wait for it
   // (and every earlier grid of the stream) before reading any global memory.
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (blockIdx.y == gridDim.y - 1) {
+    // Schedule the next pass while the other blocks apply this one: it reads
+    // the entry table this pass already produced and writes the other buffer.
+    __shared__ SchedShared sched;
+    if (a.la_out != nullptr && blockIdx.x == 0 && threadIdx.x < 32)
+      schedule_pass(sched, a.la_in, a.la_out, a.status, a.la_frames, a.M, a.la_beta, a.la_anchor, a.la_op,
+                    a.la_expected);
+    return;
+  }
   const DevPlan& p = a.st->plan;
   if (threadIdx.x < kMaxSrc) {
     s_ref[threadIdx.x] = p.src_ref[threadIdx.x];
@@ -337,6 +368,10 @@ __global__ void __launch_bounds__(256) consolidate_kernel(const __grid_constant_
   }
   if (threadIdx.x < kMaxDest) s_dslot[threadIdx.x] = p.dest_slot[threadIdx.x];
   if (threadIdx.x == 0) s_ns = p.n_src;
+  if (threadIdx.x == 0 && blockIdx.x == 0 && blockIdx.y == 0) {
+    atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
+    atomicAdd(&a.totals[1], 1ull);
+  }
   __syncthreads();
   const int ns = s_ns;
   if (ns == 0) return;
@@ -392,17 +427,26 @@ __global__ void __launch_bounds__(256) consolidate_kernel(const __grid_constant_
 
 }  // namespace
 
-cudaError_t launch_schedule(DevState* st, int frames, int M, double beta, int anchor, int op, int expected_count,
-                            cudaStream_t stream) {
+cudaError_t launch_schedule(const DevState* in, DevState* out, unsigned int* status, int frames, int M, double beta,
+                            int anchor, int op, int expected_count, cudaStream_t stream) {
   if (frames < 1 || frames > kMaxPassFrames) return cudaErrorInvalidValue;
-  schedule_kernel<<<1, 32, 0, stream>>>(st, frames, M, beta, anchor, op, expected_count);
+  schedule_kernel<<<1, 32, 0, stream>>>(in, out, status, frames, M, beta, anchor, op, expected_count);
   return cudaGetLastError();
 }
 
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
-                               int frames, int op, cudaStream_t stream) {
+                               int frames, int op, const Lookahead& la, cudaStream_t stream) {
   (void)frames;
   ConsolidateArgs a;
+  a.la_in = la.in;
+  a.la_out = la.out;
+  a.status = la.status;
+  a.totals = la.totals;
+  a.la_frames = la.frames;
+  a.la_expected = la.expected_count;
+  a.la_anchor = la.anchor;
+  a.la_op = la.op;
+  a.la_beta = la.beta;
   a.cache = reinterpret_cast<char*>(cache_base);
   a.st = st;
   a.L = g.L; a.H = g.H; a.M = g.M; a.N = g.N; a.D = g.D;
@@ -416,9 +460,21 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   a.srcs = srcs;
   const int nvec = g.N * dv;
   const int threads = 256;
-  int bx = (nvec + threads * 2 - 1) / (threads * 2);
+  // One wave: (SMs x resident blocks) spread evenly over the layer*K|V*head rows;
+  // each thread then strides over its row's vectors.
+  static int num_sms = 0;
+  if (num_sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                   cudaSuccess)
+      num_sms = 148;
+  }
+  const int rows = g.L * 2 * g.H;
+  int bx = (num_sms * kConsolidateBlocksPerSM) / rows;
+  const int bx_max = (nvec + threads - 1) / threads;
+  if (bx > bx_max) bx = bx_max;
   if (bx < 1) bx = 1;
-  dim3 grid(bx, g.L * 2 * g.H);
+  dim3 grid(bx, rows + 1);  // + one row for the lookahead schedule
   const bool mx = op == FADEMEM_MERGE_MAX_POOL;
   void (*kern)(const ConsolidateArgs);
   if (g.dtype == FADEMEM_BF16)

@@ -47,9 +47,17 @@ struct fademem_ctx {
   Geometry g;
   char* ws;
   size_t ws_bytes;
-  DevState* st;
+  unsigned int* status;  // device status word (workspace)
+  DevState* st_buf[2];   // two entry-table buffers (workspace)
+  int cur;               // st_buf[cur] holds the current entry table
   char* cache;
   bool need_init;
+  // Schedule lookahead: the consolidation kernel of a single-pass call also
+  // schedules the next pass (assuming as many frames) into st_buf[1 - cur].
+  bool la_valid;         // st_buf[1 - cur] holds that plan
+  int la_frames;         // the frame count it assumed
+  bool la_enabled;
+  unsigned long long launches = 0;  // kernels this handle launched
   int count;             // entries, = min(frames, M) (one merge per insert beyond the budget)
   long long frames;      // consolidated frames
   std::vector<Chunk> pending[FADEMEM_MAX_LAYERS];
@@ -88,7 +96,7 @@ static fademem_status check_config(const fademem_config* c, Geometry* g) {
     g->elem = c->dtype == FADEMEM_BF16 ? 2 : 4;
     g->slab_elems = (size_t)g->N * g->D;
     g->kv_elems = (size_t)g->H * g->M * g->slab_elems;
-    g->state_bytes = round_up(sizeof(DevState), 256);
+    g->state_bytes = 256 + 2 * round_up(sizeof(DevState), 256);
     g->layer_bytes = round_up(2 * g->kv_elems * g->elem, 256);
     g->total_bytes = g->state_bytes + (size_t)g->L * g->layer_bytes;
   }
@@ -122,8 +130,14 @@ FADEMEM_API fademem_status fademem_create(const fademem_config* cfg, void* works
   h->g = g;
   h->ws = reinterpret_cast<char*>(workspace);
   h->ws_bytes = workspace_bytes;
-  h->st = reinterpret_cast<DevState*>(h->ws);
+  h->status = reinterpret_cast<unsigned int*>(h->ws);
+  h->st_buf[0] = reinterpret_cast<DevState*>(h->ws + 256);
+  h->st_buf[1] = reinterpret_cast<DevState*>(h->ws + 256 + round_up(sizeof(DevState), 256));
+  h->cur = 0;
   h->cache = h->ws + g.state_bytes;
+  h->la_valid = false;
+  h->la_frames = 0;
+  h->la_enabled = true;
   h->need_init = true;
   h->count = 0;
   h->frames = 0;
@@ -146,13 +160,18 @@ FADEMEM_API fademem_status fademem_insert(fademem_t h, int layer, const void* K,
   return FADEMEM_OK;
 }
 
+static DevState* cur_state(fademem_t h) { return h->st_buf[h->cur]; }
+
 static fademem_status ensure_init(fademem_t h, cudaStream_t stream) {
   if (!h->need_init) return FADEMEM_OK;
-  cudaError_t e = cudaMemsetAsync(h->st, 0, sizeof(DevState), stream);
+  cudaError_t e = cudaMemsetAsync(h->ws, 0, h->g.state_bytes, stream);
   if (e != cudaSuccess) return cuda_fail(e, "initialising the entry table");
+  h->cur = 0;
   h->need_init = false;
   return FADEMEM_OK;
 }
+
+
 
 FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
@@ -168,28 +187,69 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   if (s != FADEMEM_OK) return s;
 
   const size_t frame_bytes = (size_t)h->g.N * h->g.H * h->g.D * h->g.elem;
+  // Passes: at most kMaxPassFrames frames each, never crossing an insert boundary.
+  std::vector<int> pass_frames;
+  {
+    std::vector<int> ci(L, 0), co(L, 0);
+    int done = 0;
+    while (done < F) {
+      int nf = F - done < kMaxPassFrames ? F - done : kMaxPassFrames;
+      for (int l = 0; l < L; ++l) {
+        const int left = h->pending[l][ci[l]].frames - co[l];
+        if (left < nf) nf = left;
+      }
+      pass_frames.push_back(nf);
+      for (int l = 0; l < L; ++l) {
+        co[l] += nf;
+        if (co[l] == h->pending[l][ci[l]].frames) {
+          ++ci[l];
+          co[l] = 0;
+        }
+      }
+      done += nf;
+    }
+  }
+  // A lookahead schedule fits if it assumed exactly this single pass; it was
+  // written by an earlier kernel on this stream, so stream order suffices.
+  const bool use_la = h->la_valid && pass_frames.size() == 1 && pass_frames[0] == h->la_frames;
+  h->la_valid = false;
+  const bool make_la = h->la_enabled && pass_frames.size() == 1;
   std::vector<int> ci(L, 0), co(L, 0);  // chunk index and frame offset inside it, per layer
   PassSources srcs;
   memset(&srcs, 0, sizeof(srcs));
-  int done = 0;
-  while (done < F) {
-    int nf = F - done < kMaxPassFrames ? F - done : kMaxPassFrames;
-    for (int l = 0; l < L; ++l) {
-      const int left = h->pending[l][ci[l]].frames - co[l];
-      if (left < nf) nf = left;  // a pass never crosses an insert boundary
-    }
+  for (size_t pi = 0; pi < pass_frames.size(); ++pi) {
+    const int nf = pass_frames[pi];
     for (int l = 0; l < L; ++l) {
       const Chunk& c = h->pending[l][ci[l]];
       srcs.src[l][0] = c.K + (size_t)co[l] * frame_bytes;
       srcs.src[l][1] = c.V + (size_t)co[l] * frame_bytes;
     }
-    cudaError_t e = launch_schedule(h->st, nf, h->g.M, h->cfg.beta, h->cfg.anchor, h->cfg.merge_op, h->count,
-                                    stream);
-    if (e != cudaSuccess) return cuda_fail(e, "launching the schedule kernel");
-    e = launch_consolidate(h->g, h->cache, h->st, srcs, nf, h->cfg.merge_op, stream);
+    cudaError_t e;
+    if (pi == 0 && use_la) {
+      h->cur ^= 1;  // the lookahead already wrote this pass's entry table and plan
+    } else {
+      e = launch_schedule(cur_state(h), cur_state(h), h->status, nf, h->g.M, h->cfg.beta, h->cfg.anchor,
+                          h->cfg.merge_op, h->count, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "launching the schedule kernel");
+      ++h->launches;
+    }
+    const long long frames_after = h->frames + nf;
+    const int count_after = frames_after < h->g.M ? (int)frames_after : h->g.M;
+    Lookahead la;
+    la.in = cur_state(h);
+    la.out = make_la ? h->st_buf[h->cur ^ 1] : nullptr;
+    la.status = h->status;
+    la.totals = reinterpret_cast<unsigned long long*>(h->ws + 8);
+    la.frames = nf;
+    la.expected_count = count_after;
+    la.anchor = h->cfg.anchor;
+    la.op = h->cfg.merge_op;
+    la.beta = h->cfg.beta;
+    e = launch_consolidate(h->g, h->cache, cur_state(h), srcs, nf, h->cfg.merge_op, la, stream);
     if (e != cudaSuccess) return cuda_fail(e, "launching the consolidation kernel");
-    h->frames += nf;
-    h->count = h->frames < h->g.M ? (int)h->frames : h->g.M;
+    ++h->launches;
+    h->frames = frames_after;
+    h->count = count_after;
     for (int l = 0; l < L; ++l) {
       co[l] += nf;
       if (co[l] == h->pending[l][ci[l]].frames) {
@@ -197,11 +257,14 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
         co[l] = 0;
       }
     }
-    done += nf;
   }
   for (int l = 0; l < L; ++l) {
     h->pending[l].clear();
     h->pending_frames[l] = 0;
+  }
+  if (make_la) {
+    h->la_valid = true;
+    h->la_frames = F;
   }
   return FADEMEM_OK;
 }
@@ -231,12 +294,13 @@ static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const v
                           reinterpret_cast<float*>(out), Lq, h->cfg.scale, stream);
   } else {
     char msg[256] = "";
-    e = launch_attend_bf16(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, Q, out, Lq, h->cfg.scale, &h->st->status, stream, msg,
+    e = launch_attend_bf16(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, Q, out, Lq, h->cfg.scale, h->status, stream, msg,
                            sizeof(msg));
     if (e == cudaErrorNotSupported) return fail(FADEMEM_ERR_UNSUPPORTED, "%s", msg);
     if (e == cudaErrorInvalidValue && msg[0]) return fail(FADEMEM_ERR_INVALID_ARG, "%s", msg);
   }
   if (e != cudaSuccess) return cuda_fail(e, "launching the attention kernel");
+  ++h->launches;
   return FADEMEM_OK;
 }
 
@@ -267,7 +331,7 @@ FADEMEM_API fademem_status fademem_get_entries(fademem_t h, void* stream_, int c
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
   DevMeta m;
-  e = cudaMemcpy(&m, &h->st->meta, sizeof(m), cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(&m, &cur_state(h)->meta, sizeof(m), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "reading the entry table");
   if (m.count < 0 || m.count > kMaxEntries)
     return fail(FADEMEM_ERR_DEVICE_CHECK, "device entry count %d is out of range", m.count);
@@ -290,11 +354,28 @@ FADEMEM_API fademem_status fademem_last_plan(fademem_t h, void* stream_, int* n_
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
   DevPlan p;
-  e = cudaMemcpy(&p, &h->st->plan, sizeof(p), cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(&p, &cur_state(h)->plan, sizeof(p), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "reading the merge plan");
   if (n_src) *n_src = p.n_src;
   if (n_dest) *n_dest = p.n_dest;
   if (frames) *frames = p.frames;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_stats(fademem_t h, void* stream_, uint64_t* blocks_moved, uint64_t* passes,
+                                        uint64_t* kernel_launches) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  unsigned long long t[2] = {0, 0};
+  e = cudaMemcpy(t, h->ws + 8, sizeof(t), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the consolidation counters");
+  if (blocks_moved) *blocks_moved = t[0];
+  if (passes) *passes = t[1];
+  if (kernel_launches) *kernel_launches = h->launches;
   return FADEMEM_OK;
 }
 
@@ -315,10 +396,10 @@ FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void* stream_,
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
   unsigned int w = 0;
-  e = cudaMemcpy(&w, &h->st->status, sizeof(w), cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(&w, h->status, sizeof(w), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "reading the device status");
   const unsigned int zero = 0;
-  e = cudaMemcpy(&h->st->status, &zero, sizeof(zero), cudaMemcpyHostToDevice);
+  e = cudaMemcpy(h->status, &zero, sizeof(zero), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
   if (word) *word = w;
   if (w & kStatusTimeout) return fail(FADEMEM_ERR_DEVICE_TIMEOUT, "a device wait timed out (status 0x%x)", w);
@@ -331,13 +412,15 @@ FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void* stre
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   fademem_status s = ensure_init(h, stream);
   if (s != FADEMEM_OK) return s;
-  cudaError_t e = launch_wait_selftest(&h->st->status, 2000000LL, stream);  // about 1 ms
+  cudaError_t e = launch_wait_selftest(h->status, 2000000LL, stream);  // about 1 ms
   if (e != cudaSuccess) return cuda_fail(e, "launching the wait self-test");
+  ++h->launches;
   return FADEMEM_OK;
 }
 
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->la_valid = false;
   h->need_init = true;
   fademem_status s = ensure_init(h, reinterpret_cast<cudaStream_t>(stream_));
   if (s != FADEMEM_OK) return s;
@@ -397,13 +480,18 @@ FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream
   if (s != FADEMEM_OK) return s;
   s = ensure_init(h, stream);
   if (s != FADEMEM_OK) return s;
-  cudaError_t e = cudaMemcpyAsync(scratch, h->st, sizeof(DevState), cudaMemcpyDeviceToDevice, stream);
+  // A lookahead schedule lives in the workspace's second entry-table buffer:
+  // drop it, and schedule in place on the scratch copy instead.
+  h->la_valid = false;
+  DevState* own = cur_state(h);
+  cudaError_t e = cudaMemcpyAsync(scratch, own, sizeof(DevState), cudaMemcpyDeviceToDevice, stream);
   if (e != cudaSuccess) return cuda_fail(e, "copying the entry table to the no-alloc scratch");
   // Run the ordinary consolidation on the scratch copy, then copy the result back.
-  DevState* own = h->st;
-  h->st = scratch;
+  h->st_buf[h->cur] = scratch;
+  h->la_enabled = false;
   const fademem_status rs = fademem_consolidate(h, stream_);
-  h->st = own;
+  h->la_enabled = true;
+  h->st_buf[h->cur] = own;
   e = cudaMemcpyAsync(own, scratch, sizeof(DevState), cudaMemcpyDeviceToDevice, stream);
   if (rs != FADEMEM_OK) return rs;
   if (e != cudaSuccess) return cuda_fail(e, "copying the entry table back from the no-alloc scratch");

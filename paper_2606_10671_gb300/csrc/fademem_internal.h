@@ -52,8 +52,6 @@ struct DevPlan {
 struct DevState {
   DevMeta meta;
   DevPlan plan;
-  unsigned int status;
-  unsigned int pad[7];
 };
 
 // Layout of one layer in the workspace: K then V, each [H][M][N][D].
@@ -63,7 +61,7 @@ struct Geometry {
   size_t elem;           // bytes per element
   size_t slab_elems;     // N * D
   size_t kv_elems;       // H * M * N * D (one of K or V of one layer)
-  size_t state_bytes;    // DevState, rounded to 256
+  size_t state_bytes;    // status word + two DevState buffers, each rounded to 256
   size_t layer_bytes;    // 2 * kv_elems * elem, rounded to 256
   size_t total_bytes;
 };
@@ -74,12 +72,24 @@ struct PassSources {
   const void* src[FADEMEM_MAX_LAYERS][2];
 };
 
-// expected_count: the host's entry count before the pass (count = min(frames, M));
-// a mismatch sets kStatusCountMismatch in the device status word.
-cudaError_t launch_schedule(DevState* st, int frames, int M, double beta, int anchor, int op, int expected_count,
-                            cudaStream_t stream);
+// Schedules one pass of `frames` units: reads in->meta, writes out->meta and
+// out->plan (in == out for an in-place pass).  expected_count: the host's
+// entry count before the pass (count = min(frames, M)); a mismatch sets
+// kStatusCountMismatch in *status and leaves an empty plan.
+cudaError_t launch_schedule(const DevState* in, DevState* out, unsigned int* status, int frames, int M, double beta,
+                            int anchor, int op, int expected_count, cudaStream_t stream);
+// Schedule of the next pass computed inside the consolidation kernel (by one
+// extra block) from the entry table `in` into `out`; out == nullptr skips it.
+struct Lookahead {
+  const DevState* in;
+  DevState* out;
+  unsigned int* status;
+  unsigned long long* totals;  // consolidation counters: [blocks moved, passes]
+  int frames, expected_count, anchor, op;
+  double beta;
+};
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
-                               int frames, int op, cudaStream_t stream);
+                               int frames, int op, const Lookahead& la, cudaStream_t stream);
 // Attention over Lk memory keys (Kc/Vc: one layer's [H][M][N][D] memory) followed
 // by Lk2 current-chunk keys (Kcur/Vcur: [Lk2][H][D]); either count may be 0.
 cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,

@@ -192,3 +192,50 @@ def test_attend_with_current_chunk_full_size():
     Kc, Vc = p.chunk(4680, step=1)
     rows = np.array([0, 5, 1234, 4095, 4679])
     p.check_attend_ext(p.queries(4680, step=9), Kc, Vc, rows=rows)
+
+
+def test_varying_frames_and_reset_with_lookahead():
+    """The next pass is scheduled ahead assuming as many frames as the last one; calls
+    with other counts (and multi-pass calls) must discard that and still match the
+    oracle, before and after a reset."""
+    p = Pair(5, 2, 64, 8, beta=0.3, dtype=torch.float32, seed=12)
+    for F in [3, 3, 3, 2, 1, 1, 4, 4, 3, 5, 3, 3, 2, 7, 2, 2]:
+        p.step(F)
+        p.check_entries()
+        p.check_memory()
+    p.check_attend(p.queries(30))
+    p.gpu.reset()
+    fresh = Pair(5, 2, 64, 8, beta=0.3, dtype=torch.float32, seed=13)
+    p.ora = fresh.ora
+    p.gens = fresh.gens
+    p.rounds = {}
+    for F in [3, 3, 1, 3, 3]:
+        p.step(F)
+        p.check_entries()
+        p.check_memory()
+    p.gpu.device_status()
+
+
+def test_stats_count_blocks_passes_and_launches():
+    """fademem_stats: blocks moved = the sum of every pass's plan (sources + written
+    slots); one consolidation kernel per pass, plus a schedule kernel only when the
+    next pass was not scheduled ahead (first pass, or a frame count that changed)."""
+    p = Pair(6, 2, 64, 8, beta=0.3, dtype=torch.float32, seed=14)
+    b0, n0, k0 = p.gpu.stats()
+    assert (b0, n0) == (0, 0)
+    blocks = 0
+    seq = [3, 3, 3, 2, 2, 4, 4, 4]
+    for F in seq:
+        p.step(F)
+        p.check_entries()
+        ns, nd, frames = p.gpu.last_plan()
+        assert frames == F
+        blocks += ns + nd
+    b1, n1, k1 = p.gpu.stats()
+    assert b1 == blocks and n1 == len(seq)
+    assert k1 - k0 == len(seq) + 3  # schedule kernels at F = 3 (first), 2 and 4
+    p.check_attend(p.queries(16))
+    assert p.gpu.stats()[2] == k1 + 1
+    p.gpu.reset()
+    assert p.gpu.stats()[:2] == (0, 0)
+    p.gpu.device_status()
