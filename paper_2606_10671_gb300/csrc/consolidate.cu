@@ -328,14 +328,15 @@ struct ConsolidateArgs {
   size_t slab_elems;      // N * D
   size_t kv_elems;        // H * M * N * D
   size_t layer_elems;     // stride between layers, in elements
-  // Lookahead: the last row of the grid (one block) schedules the next pass of
-  // la_frames units from la_in's entry table into la_out (skipped if null).
+  // Lookahead: block 0 of the grid schedules the next pass of la_frames units
+  // from la_in's entry table into la_out (skipped if null).
   const DevState* la_in;
   DevState* la_out;
   unsigned int* status;
   unsigned long long* totals;  // [blocks moved, passes] since the memory was created
   int la_frames, la_expected, la_anchor, la_op;
   double la_beta;
+  int bx;                 // blocks per (layer, K|V, head) row
   PassSources srcs;
 };
 
@@ -351,15 +352,18 @@ __global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kern
   // Launched as a programmatic dependent of the schedule kernel: wait for it
   // (and every earlier grid of the stream) before reading any global memory.
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  if (blockIdx.y == gridDim.y - 1) {
+  if (blockIdx.x == 0) {
     // Schedule the next pass while the other blocks apply this one: it reads
     // the entry table this pass already produced and writes the other buffer.
+    // Block 0 is dispatched first, so the schedule overlaps the whole copy.
     __shared__ SchedShared sched;
-    if (a.la_out != nullptr && blockIdx.x == 0 && threadIdx.x < 32)
+    if (a.la_out != nullptr && threadIdx.x < 32)
       schedule_pass(sched, a.la_in, a.la_out, a.status, a.la_frames, a.M, a.la_beta, a.la_anchor, a.la_op,
                     a.la_expected);
     return;
   }
+  const int bx = (int)(blockIdx.x - 1) % a.bx;  // block within its row
+  const int slab = (int)(blockIdx.x - 1) / a.bx;  // row: (l * 2 + kv) * H + h
   const DevPlan& p = a.st->plan;
   if (threadIdx.x < kMaxSrc) {
     s_ref[threadIdx.x] = p.src_ref[threadIdx.x];
@@ -368,7 +372,7 @@ __global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kern
   }
   if (threadIdx.x < kMaxDest) s_dslot[threadIdx.x] = p.dest_slot[threadIdx.x];
   if (threadIdx.x == 0) s_ns = p.n_src;
-  if (threadIdx.x == 0 && blockIdx.x == 0 && blockIdx.y == 0) {
+  if (threadIdx.x == 0 && blockIdx.x == 1) {
     atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
     atomicAdd(&a.totals[1], 1ull);
   }
@@ -376,7 +380,6 @@ __global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kern
   const int ns = s_ns;
   if (ns == 0) return;
 
-  const int slab = blockIdx.y;  // (l * 2 + kv) * H + h
   const int h = slab % a.H;
   const int kv = (slab / a.H) & 1;
   const int l = slab / (2 * a.H);
@@ -387,7 +390,7 @@ __global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kern
   const int dvmask = (1 << a.dv_shift) - 1;
   const int nvec = a.N << a.dv_shift;
 
-  for (int v = blockIdx.x * blockDim.x + threadIdx.x; v < nvec; v += gridDim.x * blockDim.x) {
+  for (int v = bx * blockDim.x + threadIdx.x; v < nvec; v += a.bx * blockDim.x) {
     const int n = v >> a.dv_shift;
     const int d = (v & dvmask) * V::kN;
     const size_t in_slab = (size_t)n * a.D + d;
@@ -474,7 +477,8 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   const int bx_max = (nvec + threads - 1) / threads;
   if (bx > bx_max) bx = bx_max;
   if (bx < 1) bx = 1;
-  dim3 grid(bx, rows + 1);  // + one row for the lookahead schedule
+  a.bx = bx;
+  dim3 grid(1 + bx * rows);  // block 0: the lookahead schedule
   const bool mx = op == FADEMEM_MERGE_MAX_POOL;
   void (*kern)(const ConsolidateArgs);
   if (g.dtype == FADEMEM_BF16)
