@@ -172,6 +172,18 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
       : "memory");
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// Wait for this thread's outstanding TMEM loads, with r as an in/out operand
+// so that no use of the loaded registers is scheduled before the wait.
+__device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 // Shared-memory matrix descriptor, 128-byte swizzle (tcgen05 format: start,
@@ -223,6 +235,32 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 b = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&b);
+}
+
+// Row-sum bound of the softmax fast path: every exponential of the row is at
+// most the sum, so P stays far inside bf16/fp32 range.
+constexpr float kFastRowSumLimit = 65536.f;
+
+// Exponentials of one quarter (32 keys) of this thread's row of S:
+// x = s * scale_log2 + neg_m, e = 2^x (0 for keys past `valid`), summed into
+// (rs0, rs1) and packed as bf16 pairs into pk[16 qtr .. 16 qtr + 15].
+// kRagged masks the keys past `valid` (the last tile of either key source).
+template <bool kRagged>
+__device__ __forceinline__ void exp_quarter(const uint32_t (&r)[32], int qtr, int valid, float scale_log2,
+                                            float neg_m, float& rs0, float& rs1, uint32_t (&pk)[64]) {
+#pragma unroll
+  for (int c = 0; c < 32; c += 2) {
+    float x0, x1;
+    ffma2(x0, x1, __uint_as_float(r[c]), __uint_as_float(r[c + 1]), scale_log2, scale_log2, neg_m, neg_m);
+    if (kRagged) {
+      if (32 * qtr + c >= valid) x0 = -INFINITY;
+      if (32 * qtr + c + 1 >= valid) x1 = -INFINITY;
+    }
+    const float e0 = ex2(x0);
+    const float e1 = ex2(x1);
+    fadd2(rs0, rs1, rs0, rs1, e0, e1);
+    pk[16 * qtr + c / 2] = pack_bf16(e0, e1);
+  }
 }
 
 __device__ __forceinline__ uint32_t barat(uint32_t bar0, int i) { return bar0 + 8u * (uint32_t)i; }
@@ -420,66 +458,75 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         if (j >= 2) mbar_arrive(barat(bar0, BAR_VEMPTY + (j - 2) % kVStages));
       }
       tc_fence_after();
-      float sv[kBN];
-      {
-        uint32_t r0[32], r1[32], r2[32], r3[32];
-        tmem_ld32(tS, r0);
-        tmem_ld32(tS + 32, r1);
-        tmem_ld32(tS + 64, r2);
-        tmem_ld32(tS + 96, r3);
-        tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          sv[i] = __uint_as_float(r0[i]);
-          sv[32 + i] = __uint_as_float(r1[i]);
-          sv[64 + i] = __uint_as_float(r2[i]);
-          sv[96 + i] = __uint_as_float(r3[i]);
-        }
-      }
       const int valid = j < n1 ? p.Lk - j * kBN : p.Lk2 - (j - n1) * kBN;  // keys of this tile
-      if (valid < kBN) {  // the last tile of either source is ragged
-#pragma unroll
-        for (int c = 0; c < kBN; ++c)
-          if (c >= valid) sv[c] = -INFINITY;
-      }
-      float mx[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) mx[k] = fmaxf(sv[2 * k], sv[2 * k + 1]);
-#pragma unroll
-      for (int c = 16; c < kBN; c += 16)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = fmax3(mx[k], sv[c + 2 * k], sv[c + 2 * k + 1]);
-      const float mt = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) *
-                       p.scale_log2;
-      // Lazy reference maximum: move it only when the tile exceeds it by > 8 (2^8 headroom).
-      const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
-      const float m_new = move ? fmaxf(mt, m_run) : m_run;
-      const float alpha = ex2(m_run - m_new);  // 0 on the group's first tile, 1 if unchanged
+      // Fast path: exponentials against the running reference maximum m_run,
+      // with no max over the tile first.  Any reference keeps the softmax exact
+      // (it cancels in O / l) as long as no exponential overflows, and the row
+      // sum bounds every term of the row, so a sum <= 2^16 (finite, not NaN)
+      // proves the tile safe.  The TMEM load of the next quarter of S overlaps
+      // the exponentials of the current one.  P is held in registers until the
+      // check passes, so S is still intact for the slow path.
+      uint32_t pk[64];
       float rs0 = 0.f, rs1 = 0.f;
+      {
+        const float neg_m = -m_run;
+        uint32_t r[2][32];
+        tmem_ld32(tS, r[0]);
+        tmem_ld_wait_regs(r[0]);
 #pragma unroll
-      for (int qtr = 0; qtr < 4; ++qtr) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int c = 0; c < 32; c += 2) {
-          float x0, x1;
-          ffma2(x0, x1, sv[32 * qtr + c], sv[32 * qtr + c + 1], p.scale_log2, p.scale_log2, -m_new, -m_new);
-          const float e0 = ex2(x0);
-          const float e1 = ex2(x1);
-          fadd2(rs0, rs1, rs0, rs1, e0, e1);
-          pk[c / 2] = pack_bf16(e0, e1);
+        for (int qtr = 0; qtr < 4; ++qtr) {
+          if (qtr < 3) tmem_ld32(tS + 32 * (qtr + 1), r[(qtr + 1) & 1]);
+          if (valid < kBN)
+            exp_quarter<true>(r[qtr & 1], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk);
+          else
+            exp_quarter<false>(r[qtr & 1], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk);
+          if (qtr < 3) tmem_ld_wait_regs(r[(qtr + 1) & 1]);
         }
-        tmem_st16(tS + qtr * 16, pk);  // P over the first 64 columns of the S buffer
       }
+      float alpha = 1.f;
+      bool moved = false;
+      if (__any_sync(0xffffffffu, !(rs0 + rs1 <= kFastRowSumLimit))) {
+        // Slow path (a group's first tile, or a row maximum that outgrew the
+        // reference): reload S, take the tile maximum, and move the reference
+        // lazily, only when the tile exceeds it by more than 2^8.
+        uint32_t r[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, r[c]);
+        tmem_ld_wait_regs(r[0]);
+        tmem_ld_wait_regs(r[1]);
+        tmem_ld_wait_regs(r[2]);
+        tmem_ld_wait_regs(r[3]);
+        float mx = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const float s0 = 32 * c + i < valid ? __uint_as_float(r[c][i]) : -INFINITY;
+            const float s1 = 32 * c + i + 1 < valid ? __uint_as_float(r[c][i + 1]) : -INFINITY;
+            mx = fmax3(mx, s0, s1);
+          }
+        const float mt = mx * p.scale_log2;
+        const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
+        const float m_new = move ? fmaxf(mt, m_run) : m_run;
+        alpha = ex2(m_run - m_new);  // 0 on the group's first tile, 1 if unchanged
+        m_run = m_new;
+        rs0 = 0.f;
+        rs1 = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) exp_quarter<true>(r[c], c, valid, p.scale_log2, -m_new, rs0, rs1, pk);
+        moved = __any_sync(0xffffffffu, move);
+      }
+      tmem_st32(tS, *reinterpret_cast<const uint32_t(*)[32]>(&pk[0]));  // P over the first 64 columns of S
+      tmem_st32(tS + 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[32]));
       l_run = l_run * alpha + (rs0 + rs1);
-      m_run = m_new;
-      if (j >= 2 && __any_sync(0xffffffffu, move)) {
+      if (j >= 2 && moved) {
         // Rescale O_grp before P_j V_j accumulates into it.  Its last update
         // (P_{j-2} V_{j-2}) was issued before S_j, so it is complete once S_j is.
 #pragma unroll
         for (int c = 0; c < kHD / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(tO + c * 32, r);
-          tmem_ld_wait();
+          tmem_ld_wait_regs(r);
 #pragma unroll
           for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
           tmem_st32(tO + c * 32, r);

@@ -340,14 +340,27 @@ struct ConsolidateArgs {
   PassSources srcs;
 };
 
-constexpr int kConsolidateBlocksPerSM = 3;  // resident 256-thread blocks per SM (register-limited)
+// K2 geometry: one wave of 256-thread blocks, 4 per SM (64 registers a
+// thread), spread over the (layer, K|V, head) rows.  Each thread owns one
+// 16-byte vector coordinate per iteration: it loads every plan source at that
+// coordinate (all loads in flight together), then combines and stores every
+// destination.  Because each read of a coordinate precedes every write to it
+// in the same thread, slots that are both read and rewritten need no second
+// buffer.  kNS bounds the sources of the pass: F frames make at most F merges,
+// which touch at most 2F entries, plus F frame copies, so kNS = 3F suffices;
+// a larger plan is refused through the status word.
+constexpr int kConsThreads = 256;
+// Resident blocks per SM: 4 (64 registers) while the sources fit, 3 for 12.
+__host__ __device__ constexpr int cons_blocks_per_sm(int ns_max) { return ns_max <= 9 ? 4 : 3; }
 
-template <typename T, bool kMax>
-__global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kernel(
+template <typename T, bool kMax, int kNS>
+__global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consolidate_kernel(
     const __grid_constant__ ConsolidateArgs a) {
   using V = Vec<T>;
-  __shared__ int s_ref[kMaxSrc], s_dest[kMaxSrc], s_dslot[kMaxDest];
+  __shared__ const T* s_base[kMaxSrc];  // source k at token n: s_base[k] + n * (token stride) + d
+  __shared__ T* s_dst[kMaxSrc];         // destination of the run that source k ends
   __shared__ float s_w[kMaxSrc];
+  __shared__ unsigned s_frame_mask, s_end_mask;  // bit k: source k is a frame / ends its run
   __shared__ int s_ns;
   // Launched as a programmatic dependent of the schedule kernel: wait for it
   // (and every earlier grid of the stream) before reading any global memory.
@@ -362,66 +375,88 @@ __global__ void __launch_bounds__(256, kConsolidateBlocksPerSM) consolidate_kern
                     a.la_expected);
     return;
   }
-  const int bx = (int)(blockIdx.x - 1) % a.bx;  // block within its row
+  const int bx = (int)(blockIdx.x - 1) % a.bx;    // block within its row
   const int slab = (int)(blockIdx.x - 1) / a.bx;  // row: (l * 2 + kv) * H + h
-  const DevPlan& p = a.st->plan;
-  if (threadIdx.x < kMaxSrc) {
-    s_ref[threadIdx.x] = p.src_ref[threadIdx.x];
-    s_dest[threadIdx.x] = p.src_dest[threadIdx.x];
-    s_w[threadIdx.x] = p.src_w[threadIdx.x];
-  }
-  if (threadIdx.x < kMaxDest) s_dslot[threadIdx.x] = p.dest_slot[threadIdx.x];
-  if (threadIdx.x == 0) s_ns = p.n_src;
-  if (threadIdx.x == 0 && blockIdx.x == 1) {
-    atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
-    atomicAdd(&a.totals[1], 1ull);
-  }
-  __syncthreads();
-  const int ns = s_ns;
-  if (ns == 0) return;
-
   const int h = slab % a.H;
   const int kv = (slab / a.H) & 1;
   const int l = slab / (2 * a.H);
   T* cache = reinterpret_cast<T*>(a.cache) + (size_t)l * a.layer_elems + (size_t)kv * a.kv_elems +
              (size_t)h * a.M * a.slab_elems;
-  const T* frame0 = reinterpret_cast<const T*>(a.srcs.src[l][kv]);
-  const size_t frame_elems = (size_t)a.N * a.H * a.D;
-  const int dvmask = (1 << a.dv_shift) - 1;
-  const int nvec = a.N << a.dv_shift;
-
-  for (int v = bx * blockDim.x + threadIdx.x; v < nvec; v += a.bx * blockDim.x) {
-    const int n = v >> a.dv_shift;
-    const int d = (v & dvmask) * V::kN;
-    const size_t in_slab = (size_t)n * a.D + d;
-    const size_t in_frame = ((size_t)n * a.H + h) * a.D + d;
-    uint4 raw[kMaxSrc];
-#pragma unroll
-    for (int k = 0; k < kMaxSrc; ++k) {
-      if (k < ns) {
-        const int r = s_ref[k];
-        const T* src = r >= 0 ? cache + (size_t)r * a.slab_elems + in_slab
-                              : frame0 + (size_t)(-r - 1) * frame_elems + in_frame;
-        raw[k] = __ldcs(reinterpret_cast<const uint4*>(src));
+  if (threadIdx.x < 32) {
+    // The plan lists the sources of each changed slot consecutively; lane k
+    // decodes source k (all lanes at once, no dependent chain of loads).
+    const DevPlan& p = a.st->plan;
+    const int k = threadIdx.x;
+    int ns = p.n_src;
+    if (ns < 0 || ns > kMaxSrc) ns = kMaxSrc + 1;  // refused below (ns > kNS)
+    bool frame = false, end = false, bad = false;
+    if (k < ns && k < kMaxSrc) {
+      int r = p.src_ref[k];
+      int dk = p.src_dest[k];
+      if (dk < 0 || dk >= kMaxDest || r >= a.M || r < -kMaxPassFrames || p.dest_slot[dk] < 0 ||
+          p.dest_slot[dk] >= a.M) {
+        bad = true;
+        dk = 0;
+        r = 0;
+      }
+      frame = r < 0;
+      end = (k + 1 == ns) || (k + 1 < kMaxSrc && p.src_dest[k + 1] != dk);
+      s_base[k] = frame ? reinterpret_cast<const T*>(a.srcs.src[l][kv]) + (size_t)(-r - 1) * a.N * a.H * a.D +
+                              (size_t)h * a.D
+                        : cache + (size_t)r * a.slab_elems;
+      s_w[k] = p.src_w[k];
+      s_dst[k] = cache + (size_t)(bad ? 0 : p.dest_slot[dk]) * a.slab_elems;
+    }
+    const unsigned fm = __ballot_sync(0xffffffffu, frame), em = __ballot_sync(0xffffffffu, end);
+    if (__any_sync(0xffffffffu, bad)) ns = kMaxSrc + 1;
+    if (k == 0) {
+      s_frame_mask = fm;
+      s_end_mask = em;
+      s_ns = ns;
+      if (blockIdx.x == 1) {
+        atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
+        atomicAdd(&a.totals[1], 1ull);
       }
     }
+  }
+  __syncthreads();
+  const int ns = s_ns;
+  if (ns == 0) return;
+  if (ns > kNS) {
+    if (threadIdx.x == 0 && blockIdx.x == 1) atomicOr(a.status, kStatusPlanOverflow);
+    return;
+  }
+  const unsigned fmask = s_frame_mask, emask = s_end_mask;
+  const int dvmask = (1 << a.dv_shift) - 1;
+  const int nvec = a.N << a.dv_shift;
+  const unsigned frame_tok = (unsigned)(a.H * a.D);
+
+  // Offsets within one slab (< N*D) or one frame (< N*H*D < 2^31) fit in 32 bits.
+  for (int v = bx * kConsThreads + threadIdx.x; v < nvec; v += a.bx * kConsThreads) {
+    const unsigned n = (unsigned)v >> a.dv_shift;
+    const unsigned d = (unsigned)(v & dvmask) * V::kN;
+    const unsigned off_slab = n * (unsigned)a.D + d;
+    const unsigned off_frame = n * frame_tok + d;
+    uint4 raw[kNS];
+#pragma unroll
+    for (int k = 0; k < kNS; ++k)
+      if (k < ns)
+        raw[k] = __ldcs(reinterpret_cast<const uint4*>(s_base[k] + ((fmask >> k) & 1 ? off_frame : off_slab)));
     float acc[V::kN];
 #pragma unroll
-    for (int k = 0; k < kMaxSrc; ++k) {
+    for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? -INFINITY : 0.f;
+#pragma unroll
+    for (int k = 0; k < kNS; ++k) {
       if (k < ns) {
         float x[V::kN];
         V::unpack(raw[k], x);
-        const bool first = (k == 0) || (s_dest[k - 1] != s_dest[k]);
         const float w = s_w[k];
 #pragma unroll
-        for (int e = 0; e < V::kN; ++e) {
-          if (kMax) acc[e] = first ? x[e] : fmaxf(acc[e], x[e]);
-          else acc[e] = first ? w * x[e] : fmaf(w, x[e], acc[e]);
-        }
-        const bool last = (k + 1 == ns) || (s_dest[k + 1] != s_dest[k]);
-        if (last) {
-          T* dst = cache + (size_t)s_dslot[s_dest[k]] * a.slab_elems + in_slab;
-          *reinterpret_cast<uint4*>(dst) = V::pack(acc);
+        for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? fmaxf(acc[e], x[e]) : fmaf(w, x[e], acc[e]);
+        if ((emask >> k) & 1) {
+          *reinterpret_cast<uint4*>(s_dst[k] + off_slab) = V::pack(acc);
+#pragma unroll
+          for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? -INFINITY : 0.f;
         }
       }
     }
@@ -439,7 +474,7 @@ cudaError_t launch_schedule(const DevState* in, DevState* out, unsigned int* sta
 
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
                                int frames, int op, const Lookahead& la, cudaStream_t stream) {
-  (void)frames;
+  static_assert(kMaxSrc == 3 * kMaxPassFrames, "a pass of F frames has at most 3F sources");
   ConsolidateArgs a;
   a.la_in = la.in;
   a.la_out = la.out;
@@ -462,7 +497,6 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   a.layer_elems = g.layer_bytes / g.elem;
   a.srcs = srcs;
   const int nvec = g.N * dv;
-  const int threads = 256;
   // One wave: (SMs x resident blocks) spread evenly over the layer*K|V*head rows;
   // each thread then strides over its row's vectors.
   static int num_sms = 0;
@@ -472,22 +506,28 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
                                                    cudaSuccess)
       num_sms = 148;
   }
+  const int nsb = frames <= 2 ? 0 : frames == 3 ? 1 : 2;  // sources <= 3F: 6, 9 or 12
   const int rows = g.L * 2 * g.H;
-  int bx = (num_sms * kConsolidateBlocksPerSM) / rows;
-  const int bx_max = (nvec + threads - 1) / threads;
+  int bx = (num_sms * cons_blocks_per_sm(6 + 3 * nsb) - 1) / rows;  // - 1: the lookahead block
+  const int bx_max = (nvec + kConsThreads - 1) / kConsThreads;
   if (bx > bx_max) bx = bx_max;
   if (bx < 1) bx = 1;
   a.bx = bx;
   dim3 grid(1 + bx * rows);  // block 0: the lookahead schedule
   const bool mx = op == FADEMEM_MERGE_MAX_POOL;
-  void (*kern)(const ConsolidateArgs);
-  if (g.dtype == FADEMEM_BF16)
-    kern = mx ? consolidate_kernel<__nv_bfloat16, true> : consolidate_kernel<__nv_bfloat16, false>;
-  else
-    kern = mx ? consolidate_kernel<float, true> : consolidate_kernel<float, false>;
+  using Kern = void (*)(const ConsolidateArgs);
+  static const Kern kerns[2][2][3] = {
+      {{consolidate_kernel<float, false, 6>, consolidate_kernel<float, false, 9>,
+        consolidate_kernel<float, false, 12>},
+       {consolidate_kernel<float, true, 6>, consolidate_kernel<float, true, 9>, consolidate_kernel<float, true, 12>}},
+      {{consolidate_kernel<__nv_bfloat16, false, 6>, consolidate_kernel<__nv_bfloat16, false, 9>,
+        consolidate_kernel<__nv_bfloat16, false, 12>},
+       {consolidate_kernel<__nv_bfloat16, true, 6>, consolidate_kernel<__nv_bfloat16, true, 9>,
+        consolidate_kernel<__nv_bfloat16, true, 12>}}};
+  const Kern kern = kerns[g.dtype == FADEMEM_BF16 ? 1 : 0][mx ? 1 : 0][nsb];
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(threads);
+  cfg.blockDim = dim3(kConsThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];

@@ -86,6 +86,8 @@ static fademem_status check_config(const fademem_config* c, Geometry* g) {
     return fail(FADEMEM_ERR_UNSUPPORTED, "bf16 storage supports head_dim 128 only");
   const long long lk = (long long)c->budget * c->tokens_per_frame;
   if (lk > (1LL << 30)) return fail(FADEMEM_ERR_INVALID_ARG, "budget * tokens_per_frame too large");
+  if ((long long)c->tokens_per_frame * c->heads * c->head_dim >= (1LL << 31))
+    return fail(FADEMEM_ERR_INVALID_ARG, "tokens_per_frame * heads * head_dim must be below 2^31");
   if (g) {
     g->L = c->num_layers;
     g->H = c->heads;
