@@ -222,6 +222,37 @@ FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
  * with FADEMEM_ERR_UNSUPPORTED.  Other errors as fademem_consolidate. */
 FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void *stream);
 
+/* Device staging bytes fademem_step_host needs for segments of `nframes`
+ * frames per layer and `Lq` query tokens: two slots of the inputs (K and V
+ * of every layer, Q) plus one output block.  0 if cfg is invalid or
+ * nframes/Lq out of range.  No CUDA call is made. */
+FADEMEM_API size_t fademem_host_staging_bytes(const fademem_config *cfg, int nframes, int Lq);
+
+/* One step of a serving loop with the inputs and the result in HOST memory:
+ * copy the segment's frames and the queries in, insert the frames on every
+ * layer, consolidate (Algorithm S1 and the merges of Sec. 3.3), attend the
+ * queries over `layer`'s memory (Sec. 3.3, last paragraph), and copy the
+ * output back -- the same work as fademem_insert per layer +
+ * fademem_consolidate + fademem_attend, with the same results.
+ *   K_host[l], V_host[l]  per layer l < num_layers: [nframes*N][H][D] of the
+ *                         storage dtype (page-locked memory lets the copies
+ *                         run asynchronously; pageable memory also works)
+ *   Q_host                [Lq][H][D]; out_host [Lq][H][D] (written)
+ *   staging               caller-owned device memory of at least
+ *                         fademem_host_staging_bytes(cfg, nframes, Lq) bytes,
+ *                         16-byte aligned, used by this handle only and the
+ *                         same on every call with these sizes
+ * The host-to-device copies go on a stream of the handle's own and alternate
+ * between the two staging slots, so the copies of the next call overlap the
+ * work of this one.  Everything else, including the copy of the output to
+ * out_host, is enqueued on `stream`: once `stream` has synchronised, out_host
+ * holds this call's output and the host inputs of this call may be reused.
+ * Errors as fademem_insert / fademem_consolidate / fademem_attend, plus
+ * FADEMEM_ERR_WORKSPACE if staging is too small or misaligned. */
+FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void *const *K_host, const void *const *V_host,
+                                            int nframes, int layer, const void *Q_host, void *out_host, int Lq,
+                                            void *staging, size_t staging_bytes, void *stream);
+
 /* Release the handle (NULL-safe).  Does not free the caller's workspace. */
 FADEMEM_API void fademem_destroy(fademem_t h);
 

@@ -117,6 +117,32 @@ class FadeMem:
                                 out.data_ptr(), Lq, _stream_handle(stream))
         return out
 
+    def step_host(self, Ks, Vs, Q: torch.Tensor, out: torch.Tensor, layer: int = 0, stream=None) -> torch.Tensor:
+        """One serving step with host tensors: Ks[l], Vs[l] [nframes*N, H, D] per layer and Q [Lq, H, D]
+        (CPU, preferably pinned) in, out [Lq, H, D] (CPU) written once `stream` has synchronised.
+        Copies, insert, consolidate and attend all run inside the library (fademem_step_host)."""
+        c = self.cfg
+        if len(Ks) != c.num_layers or len(Vs) != c.num_layers:
+            raise ValueError(f"need K and V for each of the {c.num_layers} layers")
+        per_frame = c.tokens_per_frame * c.heads * c.head_dim
+        for X in list(Ks) + list(Vs) + [Q, out]:
+            if X.device.type != "cpu" or X.dtype != self.dtype or not X.is_contiguous():
+                raise ValueError("step_host takes contiguous CPU tensors of the memory's dtype")
+        nframes = Ks[0].numel() // per_frame
+        if any(X.numel() != nframes * per_frame for X in list(Ks) + list(Vs)) or nframes == 0:
+            raise ValueError("every K and V must hold the same whole number of frames")
+        Lq = Q.numel() // (c.heads * c.head_dim)
+        if Q.numel() != Lq * c.heads * c.head_dim or out.numel() != Q.numel():
+            raise ValueError(f"Q and out must be [Lq, {c.heads}, {c.head_dim}]")
+        nbytes = capi.fademem_host_staging_bytes(self.cfg, nframes, Lq)
+        st = getattr(self, "_staging", None)
+        if st is None or st.numel() < nbytes:
+            torch.cuda.synchronize(self.device)  # the old staging may still be in use
+            self._staging = st = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+        capi.fademem_step_host(self.handle, [K.data_ptr() for K in Ks], [V.data_ptr() for V in Vs], nframes, layer,
+                               Q.data_ptr(), out.data_ptr(), Lq, st.data_ptr(), st.numel(), _stream_handle(stream))
+        return out
+
     def counts(self):
         return capi.fademem_counts(self.handle)
 

@@ -35,7 +35,8 @@ EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fadem
            "fademem_attend_ext",
            "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_stats",
            "fademem_layer_memory", "fademem_get_device_status",
-           "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc", "fademem_destroy", "fademem_last_error")
+           "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc",
+           "fademem_host_staging_bytes", "fademem_step_host", "fademem_destroy", "fademem_last_error")
 
 
 class fademem_config(ctypes.Structure):
@@ -85,6 +86,8 @@ def load(path: str | None = None):
             "fademem_selftest_wait_timeout": (I, [P, P]),
             "fademem_reset": (I, [P, P]),
             "fademem_consolidate_noalloc": (I, [P, P]),
+            "fademem_host_staging_bytes": (ctypes.c_size_t, [cfgp, I, I]),
+            "fademem_step_host": (I, [P, ctypes.POINTER(P), ctypes.POINTER(P), I, I, P, P, I, P, ctypes.c_size_t, P]),
             "fademem_destroy": (None, [P]),
             "fademem_last_error": (ctypes.c_char_p, []),
         }
@@ -190,6 +193,21 @@ def fademem_reset(h: int, stream: int = 0):
 
 def fademem_consolidate_noalloc(h: int, stream: int = 0):
     check(load().fademem_consolidate_noalloc(ctypes.c_void_p(h), ctypes.c_void_p(stream)))
+
+
+def fademem_host_staging_bytes(cfg: fademem_config, nframes: int, Lq: int) -> int:
+    return int(load().fademem_host_staging_bytes(ctypes.byref(cfg), nframes, Lq))
+
+
+def fademem_step_host(h: int, K_host, V_host, nframes: int, layer: int, Q_host: int, out_host: int, Lq: int,
+                      staging: int, staging_bytes: int, stream: int = 0):
+    """K_host, V_host: sequences of host addresses, one per layer."""
+    n = len(K_host)
+    Ks = (ctypes.c_void_p * n)(*K_host)
+    Vs = (ctypes.c_void_p * n)(*V_host)
+    check(load().fademem_step_host(ctypes.c_void_p(h), Ks, Vs, nframes, layer, ctypes.c_void_p(Q_host),
+                                   ctypes.c_void_p(out_host), Lq, ctypes.c_void_p(staging), staging_bytes,
+                                   ctypes.c_void_p(stream)))
 
 
 def fademem_destroy(h: int):

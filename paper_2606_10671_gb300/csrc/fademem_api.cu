@@ -58,6 +58,13 @@ struct fademem_ctx {
   int la_frames;         // the frame count it assumed
   bool la_enabled;
   unsigned long long launches = 0;  // kernels this handle launched
+  // fademem_step_host: the copy stream, and per staging slot the events "inputs
+  // copied" and "slot no longer read by the compute stream".
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t ev_in[2] = {nullptr, nullptr};
+  cudaEvent_t ev_done[2] = {nullptr, nullptr};
+  bool done_recorded[2] = {false, false};
+  int host_slot = 0;
   int count;             // entries, = min(frames, M) (one merge per insert beyond the budget)
   long long frames;      // consolidated frames
   std::vector<Chunk> pending[FADEMEM_MAX_LAYERS];
@@ -500,7 +507,102 @@ FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream
   return FADEMEM_OK;
 }
 
-FADEMEM_API void fademem_destroy(fademem_t h) { delete h; }
+// Staging layout of fademem_step_host: slot s (s = 0, 1) holds, 256-byte
+// aligned, K then V of every layer and then Q; the output block follows both.
+struct HostStaging {
+  size_t frame_bytes, q_bytes, slot_bytes, out_off, total;
+};
+static bool host_staging(const Geometry& g, int nframes, int Lq, HostStaging* st) {
+  if (nframes < 1 || nframes > FADEMEM_MAX_PENDING || Lq < 1 || Lq > (1 << 24)) return false;
+  st->frame_bytes = round_up((size_t)nframes * g.N * g.H * g.D * g.elem, 256);
+  st->q_bytes = round_up((size_t)Lq * g.H * g.D * g.elem, 256);
+  st->slot_bytes = 2 * (size_t)g.L * st->frame_bytes + st->q_bytes;
+  st->out_off = 2 * st->slot_bytes;
+  st->total = st->out_off + st->q_bytes;
+  return true;
+}
+
+FADEMEM_API size_t fademem_host_staging_bytes(const fademem_config* cfg, int nframes, int Lq) {
+  Geometry g;
+  HostStaging st;
+  if (check_config(cfg, &g) != FADEMEM_OK || !host_staging(g, nframes, Lq, &st)) return 0;
+  return st.total;
+}
+
+FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void* const* K_host, const void* const* V_host,
+                                            int nframes, int layer, const void* Q_host, void* out_host, int Lq,
+                                            void* staging, size_t staging_bytes, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (!K_host || !V_host || !Q_host || !out_host) return fail(FADEMEM_ERR_INVALID_ARG, "a host pointer is NULL");
+  for (int l = 0; l < h->g.L; ++l)
+    if (!K_host[l] || !V_host[l]) return fail(FADEMEM_ERR_INVALID_ARG, "K_host[%d] or V_host[%d] is NULL", l, l);
+  if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
+  HostStaging st;
+  if (!host_staging(h->g, nframes, Lq, &st))
+    return fail(FADEMEM_ERR_INVALID_ARG, "nframes must be in [1, %d] and Lq in [1, 2^24]", FADEMEM_MAX_PENDING);
+  if (!staging || !aligned16(staging) || staging_bytes < st.total)
+    return fail(FADEMEM_ERR_WORKSPACE, "staging needs %zu bytes, 16-byte aligned (got %zu at %p)", st.total,
+                staging_bytes, staging);
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  cudaError_t e;
+  if (!h->copy_stream) {
+    e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
+    if (e != cudaSuccess) return cuda_fail(e, "creating the copy stream");
+    for (int s = 0; s < 2; ++s) {
+      if ((e = cudaEventCreateWithFlags(&h->ev_in[s], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&h->ev_done[s], cudaEventDisableTiming)) != cudaSuccess)
+        return cuda_fail(e, "creating the copy events");
+    }
+  }
+  const int s = h->host_slot;
+  char* slot = static_cast<char*>(staging) + s * st.slot_bytes;
+  char* dq = slot + 2 * (size_t)h->g.L * st.frame_bytes;
+  char* dout = static_cast<char*>(staging) + st.out_off;
+  const size_t fb = (size_t)nframes * h->g.N * h->g.H * h->g.D * h->g.elem;
+  const size_t qb = (size_t)Lq * h->g.H * h->g.D * h->g.elem;
+  // Inputs into slot s on the copy stream, once the compute stream is done with
+  // the slot's previous contents (the call before last).
+  if (h->done_recorded[s] && (e = cudaStreamWaitEvent(h->copy_stream, h->ev_done[s], 0)) != cudaSuccess)
+    return cuda_fail(e, "ordering the copy stream");
+  for (int l = 0; l < h->g.L; ++l) {
+    char* dk = slot + (size_t)(2 * l) * st.frame_bytes;
+    if ((e = cudaMemcpyAsync(dk, K_host[l], fb, cudaMemcpyHostToDevice, h->copy_stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dk + st.frame_bytes, V_host[l], fb, cudaMemcpyHostToDevice, h->copy_stream)) !=
+            cudaSuccess)
+      return cuda_fail(e, "copying K/V to the device");
+  }
+  if ((e = cudaMemcpyAsync(dq, Q_host, qb, cudaMemcpyHostToDevice, h->copy_stream)) != cudaSuccess)
+    return cuda_fail(e, "copying Q to the device");
+  if ((e = cudaEventRecord(h->ev_in[s], h->copy_stream)) != cudaSuccess ||
+      (e = cudaStreamWaitEvent(stream, h->ev_in[s], 0)) != cudaSuccess)
+    return cuda_fail(e, "ordering the compute stream");
+  fademem_status r;
+  for (int l = 0; l < h->g.L; ++l) {
+    char* dk = slot + (size_t)(2 * l) * st.frame_bytes;
+    if ((r = fademem_insert(h, l, dk, dk + st.frame_bytes, nframes)) != FADEMEM_OK) return r;
+  }
+  if ((r = fademem_consolidate(h, stream_)) != FADEMEM_OK) return r;
+  if ((r = fademem_attend(h, layer, dq, dout, Lq, stream_)) != FADEMEM_OK) return r;
+  if ((e = cudaMemcpyAsync(out_host, dout, qb, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    return cuda_fail(e, "copying the output to the host");
+  if ((e = cudaEventRecord(h->ev_done[s], stream)) != cudaSuccess) return cuda_fail(e, "recording the slot event");
+  h->done_recorded[s] = true;
+  h->host_slot = s ^ 1;
+  return FADEMEM_OK;
+}
+
+FADEMEM_API void fademem_destroy(fademem_t h) {
+  if (!h) return;
+  if (h->copy_stream) {
+    cudaStreamSynchronize(h->copy_stream);
+    cudaStreamDestroy(h->copy_stream);
+  }
+  for (int s = 0; s < 2; ++s) {
+    if (h->ev_in[s]) cudaEventDestroy(h->ev_in[s]);
+    if (h->ev_done[s]) cudaEventDestroy(h->ev_done[s]);
+  }
+  delete h;
+}
 
 FADEMEM_API const char* fademem_last_error(void) { return g_err; }
 

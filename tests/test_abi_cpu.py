@@ -22,7 +22,7 @@ def _declared_symbols():
 def test_exports_every_declared_symbol(cuda_lib):
     lib = ctypes.CDLL(cuda_lib)
     declared = _declared_symbols()
-    assert len(declared) == 17
+    assert len(declared) == 19
     for name in declared:
         assert hasattr(lib, name), name
     assert sorted(capi.EXPORTS) == declared
@@ -110,6 +110,44 @@ def test_host_side_call_checks(cuda_lib):
     assert (c, f) == (0, 0)
     k, v = capi.fademem_layer_memory(h, 1)
     assert v - k == 2 * 21 * 64 * 128 * 2 and k > FAKE_WS
+    capi.fademem_destroy(h)
+
+
+def test_host_step_staging_and_checks(cuda_lib):
+    """fademem_host_staging_bytes: two slots of (K, V per layer, Q) plus one output block, each
+    piece 256-byte aligned; fademem_step_host refuses bad arguments before any CUDA call."""
+    capi.load(cuda_lib)
+    lib = capi.load()
+    r = lambda x: (x + 255) // 256 * 256
+    cfg = _cfg(num_layers=2, tokens_per_frame=100, heads=3)
+    frame = r(3 * 100 * 3 * 128 * 2)  # 3 frames of K (or V), bf16
+    q = r(50 * 3 * 128 * 2)
+    assert capi.fademem_host_staging_bytes(cfg, 3, 50) == 2 * (2 * 2 * frame + q) + q
+    assert capi.fademem_host_staging_bytes(_cfg(dtype=torch.float32, num_layers=1, tokens_per_frame=7, heads=1), 1, 1) \
+        == 2 * (2 * r(7 * 128 * 4) + r(128 * 4)) + r(128 * 4)
+    for nf, lq in ((0, 50), (65, 50), (3, 0)):
+        assert capi.fademem_host_staging_bytes(cfg, nf, lq) == 0
+    assert capi.fademem_host_staging_bytes(_cfg(budget=1), 3, 50) == 0
+    st, h = _create_status(cfg)
+    assert st == capi.FADEMEM_OK
+    P = ctypes.c_void_p
+    need = capi.fademem_host_staging_bytes(cfg, 3, 50)
+    host = (ctypes.c_char * 16)()
+    hp = ctypes.addressof(host)
+    two = (P * 2)(hp, hp)
+    one_null = (P * 2)(hp, None)
+    call = lambda K=two, V=two, nf=3, layer=0, Q=hp, out=hp, lq=50, stg=FAKE_WS, nb=need: lib.fademem_step_host(
+        P(h), K, V, nf, layer, P(Q), P(out), lq, P(stg), nb, None)
+    assert call(K=one_null) == capi.FADEMEM_ERR_INVALID_ARG
+    assert call(Q=0) == capi.FADEMEM_ERR_INVALID_ARG
+    assert call(layer=2) == capi.FADEMEM_ERR_INVALID_ARG
+    assert call(nf=0) == capi.FADEMEM_ERR_INVALID_ARG
+    assert call(nb=need - 1) == capi.FADEMEM_ERR_WORKSPACE
+    assert "staging" in capi.fademem_last_error()
+    assert call(stg=FAKE_WS + 8) == capi.FADEMEM_ERR_WORKSPACE
+    assert call(stg=0) == capi.FADEMEM_ERR_WORKSPACE
+    assert lib.fademem_step_host(None, two, two, 3, 0, P(hp), P(hp), 50, P(FAKE_WS), need, None) == \
+        capi.FADEMEM_ERR_INVALID_ARG
     capi.fademem_destroy(h)
 
 

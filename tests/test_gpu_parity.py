@@ -239,3 +239,39 @@ def test_stats_count_blocks_passes_and_launches():
     p.gpu.reset()
     assert p.gpu.stats()[:2] == (0, 0)
     p.gpu.device_status()
+
+
+def test_step_host_matches_device_path():
+    """fademem_step_host (host buffers, copies inside the library, next step's copies
+    overlapping this step's work) gives bit-identical outputs and entry table to
+    insert + consolidate + attend on device buffers, over six back-to-back steps."""
+    from paper_2606_10671_gb300 import FadeMem
+    from synth import HostAR1, KIND_K, KIND_V, host_queries
+    M, H, D, N, L, F, Lq = 5, 2, 128, 100, 2, 3, 260
+    a = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=torch.bfloat16)
+    b = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=torch.bfloat16)
+    gens = [(HostAR1((N, H, D), 31 + l, KIND_K), HostAR1((N, H, D), 31 + l, KIND_V)) for l in range(L)]
+    to_bf16 = lambda x: torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(torch.bfloat16)
+    steps = []
+    for step in range(6):
+        Ks = [to_bf16(np.stack([g[0].next() for _ in range(F)])).pin_memory() for g in gens]
+        Vs = [to_bf16(np.stack([g[1].next() for _ in range(F)])).pin_memory() for g in gens]
+        Q = to_bf16(host_queries((Lq, H, D), 77, step=step)).pin_memory()
+        steps.append((Ks, Vs, Q))
+    outs_a = [torch.empty((Lq, H, D), dtype=torch.bfloat16).pin_memory() for _ in steps]
+    for (Ks, Vs, Q), out in zip(steps, outs_a):
+        a.step_host(Ks, Vs, Q, out, layer=1)
+    torch.cuda.synchronize()
+    outs_b = []
+    for Ks, Vs, Q in steps:
+        for l in range(L):
+            b.insert(l, Ks[l].cuda(), Vs[l].cuda())
+        b.consolidate()
+        outs_b.append(b.attend(1, Q.cuda()).cpu())
+    for oa, ob in zip(outs_a, outs_b):
+        assert torch.equal(oa, ob)
+    for x, y in zip(a.entries(), b.entries()):
+        assert np.array_equal(x, y)
+    assert a.counts() == b.counts() == (M, 6 * F)
+    a.device_status()
+    b.device_status()
