@@ -37,6 +37,19 @@
  *     merge happens).  This never changes what is computed.
  *   - "Select Nearest" keeps the block of the entry nearer to the current step
  *     (m_{j+1}, the smaller distance d).
+ *   - Temporal RoPE (Sec. 3.3, "Boundary and positional handling"; optional,
+ *     oracle_set_rope): the temporal band is the first P complex pairs
+ *     (dims 2k, 2k+1 for k < P) of each head's key, with the standard RoPE
+ *     frequencies omega_k = theta^(-k/P) (Su et al., the RoFormer paper the
+ *     section cites) and the rotation (x, y) -> (x cos a - y sin a,
+ *     x sin a + y cos a) by a = position * omega_k.  Keys arrive rotated to
+ *     their frame's position t; they are stored with that phase removed
+ *     (rotated by -t * omega_k).  At attention time entry i of the count
+ *     entries (temporal order) is re-indexed to position
+ *     tau_i = t_next - count + i: consecutive positions ending right before
+ *     the current chunk (frame t_next), so the exposed temporal range is
+ *     bounded by the budget M.  With no merges this gives every frame its
+ *     own position back.  Values are never rotated.
  *
  * Layout of a K or V block: elems_per_block doubles, in the caller's order.
  * For attention the order must be [token][head][dim] (tokens x heads x dim).
@@ -74,6 +87,9 @@ typedef struct oracle_memory {
     int last_j;          /* merged pair index, -1 if none */
     double last_margin;  /* (g_second - g_min) / g_second, +inf if < 2 pairs */
     double last_gmin;
+    /* temporal RoPE (0 pairs: off) */
+    int rope_pairs, rope_tokens, rope_H, rope_D;
+    double rope_theta;
 } oracle_memory;
 
 oracle_memory *oracle_create(int M, double beta, int anchor, int op, long long elems)
@@ -98,6 +114,54 @@ void oracle_destroy(oracle_memory *m)
 
 static double warp_u(double d, double beta) { return pow(d, beta); }   /* u(d) = d^beta */
 
+/* Enable temporal RoPE handling for blocks laid out [tokens][H][D]
+ * (tokens * H * D == elems), with `pairs` complex pairs (1 <= pairs <= D/2)
+ * and base theta > 1.  Call before the first insert.  Returns 0, or -1 if
+ * the arguments do not fit the memory. */
+int oracle_set_rope(oracle_memory *m, int pairs, double theta, int tokens, int H, int D)
+{
+    if (m->t_next != 0 || pairs < 1 || 2 * pairs > D || !(theta > 1.0) || tokens < 1 || H < 1 ||
+        (long long)tokens * H * D != m->elems)
+        return -1;
+    m->rope_pairs = pairs; m->rope_theta = theta;
+    m->rope_tokens = tokens; m->rope_H = H; m->rope_D = D;
+    return 0;
+}
+
+/* Rotate the temporal band of every (token, head) row of a key block by
+ * position * omega_k, in place. */
+static void rope_rotate(const oracle_memory *m, double *K, double position)
+{
+    const int P = m->rope_pairs;
+    for (int k = 0; k < P; ++k) {
+        const double a = position * pow(m->rope_theta, -(double)k / (double)P);
+        const double c = cos(a), sn = sin(a);
+        for (long long r = 0; r < (long long)m->rope_tokens * m->rope_H; ++r) {
+            double *x = K + r * m->rope_D + 2 * k;
+            const double x0 = x[0], x1 = x[1];
+            x[0] = x0 * c - x1 * sn;
+            x[1] = x0 * sn + x1 * c;
+        }
+    }
+}
+
+/* Keys of every entry as attention sees them: the stored (phase-free) keys
+ * rotated to the re-indexed positions tau_i = t_next - count + i.  Returns a
+ * malloc'd array of count * elems doubles, or NULL without RoPE (use the
+ * stored keys) or on allocation failure (*failed set). */
+static double *rope_attention_keys(const oracle_memory *m, int *failed)
+{
+    if (m->rope_pairs == 0 || m->count == 0) return NULL;
+    double *K = (double *)malloc((size_t)m->count * m->elems * sizeof(double));
+    if (!K) { *failed = 1; return NULL; }
+    for (int i = 0; i < m->count; ++i) {
+        double *Ki = K + (size_t)i * m->elems;
+        memcpy(Ki, m->e[i].K, (size_t)m->elems * sizeof(double));
+        rope_rotate(m, Ki, (double)(m->t_next - m->count + i));
+    }
+    return K;
+}
+
 /* One update of Algorithm S1.  K_t, V_t: the new unit's blocks (elems doubles
  * each; may be NULL when elems == 0, i.e. schedule-only runs).  Returns 0. */
 int oracle_insert(oracle_memory *m, const double *K_t, const double *V_t)
@@ -111,6 +175,7 @@ int oracle_insert(oracle_memory *m, const double *K_t, const double *V_t)
     nw->K = (double *)malloc(bytes ? bytes : 1);
     nw->V = (double *)malloc(bytes ? bytes : 1);
     if (bytes) { memcpy(nw->K, K_t, bytes); memcpy(nw->V, V_t, bytes); }
+    if (bytes && m->rope_pairs) rope_rotate(m, nw->K, -(double)t);   /* store without the frame's phase */
     m->count += 1;
     m->last_j = -1; m->last_margin = INFINITY; m->last_gmin = NAN;
 
@@ -208,6 +273,8 @@ int oracle_attend(const oracle_memory *m, int tokens, int H, int D,
     if ((long long)tokens * H * D != m->elems || m->count == 0) return -1;
     const long long Lk = (long long)m->count * tokens;
     int failed = 0;
+    double *Krope = rope_attention_keys(m, &failed);
+    if (failed) return -2;
 #pragma omp parallel
     {
         double *logit = (double *)malloc((size_t)Lk * sizeof(double));
@@ -224,7 +291,8 @@ int oracle_attend(const oracle_memory *m, int tokens, int H, int D,
                 long long k = 0;
                 for (int e = 0; e < m->count; ++e) {
                     for (int n = 0; n < tokens; ++n, ++k) {
-                        const double *kv = m->e[e].K + ((size_t)n * H + h) * D;
+                        const double *kv = (Krope ? Krope + (size_t)e * m->elems : m->e[e].K) +
+                                           ((size_t)n * H + h) * D;
                         double dot = 0.0;
                         for (int d = 0; d < D; ++d) dot += qv[d] * kv[d];
                         logit[k] = scale * dot;
@@ -247,6 +315,7 @@ int oracle_attend(const oracle_memory *m, int tokens, int H, int D,
         }
         free(logit);
     }
+    free(Krope);
     return failed ? -2 : 0;
 }
 
@@ -271,6 +340,8 @@ int oracle_attend_ext(const oracle_memory *m, int tokens, int H, int D, const do
     const long long Lmem = (long long)m->count * tokens;
     const long long Lk = Lmem + ncur;
     int failed = 0;
+    double *Krope = rope_attention_keys(m, &failed);
+    if (failed) return -2;
 #pragma omp parallel
     {
         double *logit = (double *)malloc((size_t)Lk * sizeof(double));
@@ -285,8 +356,12 @@ int oracle_attend_ext(const oracle_memory *m, int tokens, int H, int D, const do
                 const double *qv = Q + ((size_t)q * H + h) * D;
                 double mx = -INFINITY;
                 for (long long k = 0; k < Lk; ++k) {
-                    const double *kv = k < Lmem ? m->e[k / tokens].K + ((size_t)(k % tokens) * H + h) * D
-                                                : Kcur + ((size_t)(k - Lmem) * H + h) * D;
+                    const double *kv;
+                    if (k < Lmem)
+                        kv = (Krope ? Krope + (size_t)(k / tokens) * m->elems : m->e[k / tokens].K) +
+                             ((size_t)(k % tokens) * H + h) * D;
+                    else
+                        kv = Kcur + ((size_t)(k - Lmem) * H + h) * D;
                     double dot = 0.0;
                     for (int d = 0; d < D; ++d) dot += qv[d] * kv[d];
                     logit[k] = scale * dot;
@@ -306,5 +381,6 @@ int oracle_attend_ext(const oracle_memory *m, int tokens, int H, int D, const do
         }
         free(logit);
     }
+    free(Krope);
     return failed ? -2 : 0;
 }

@@ -61,6 +61,7 @@ def _load():
         lib.oracle_attend_ext.argtypes = [P, ctypes.c_int, ctypes.c_int, ctypes.c_int, dp, dp, ctypes.c_longlong, dp,
                                           ctypes.c_longlong, ctypes.c_double, dp]
         lib.oracle_num_threads.restype = ctypes.c_int
+        lib.oracle_set_rope.argtypes = [P, ctypes.c_int, ctypes.c_double, ctypes.c_int, ctypes.c_int, ctypes.c_int]
         _lib = lib
         return lib
 
@@ -88,6 +89,12 @@ class OracleMemory:
         if not self._h:
             raise ValueError("oracle_create rejected its arguments")
         self.budget = int(budget)
+
+    def set_rope(self, pairs: int, theta: float, tokens: int, heads: int, dim: int):
+        """Temporal RoPE handling (before the first insert): keys are stored without their
+        frame's phase and re-indexed at attention (see the C file's header)."""
+        if self._lib.oracle_set_rope(self._h, int(pairs), float(theta), int(tokens), int(heads), int(dim)) != 0:
+            raise ValueError("oracle_set_rope rejected its arguments")
 
     def close(self):
         if getattr(self, "_h", None):

@@ -344,3 +344,98 @@ def test_attention_with_current_chunk_equals_full_attention():
                                rtol=1e-12, atol=1e-13)
     none = np.zeros((0, H, D))
     np.testing.assert_array_equal(mem.attend_ext(Q, none, none, N, H, D), mem.attend(Q, N, H, D))
+
+
+# ---- temporal RoPE (Sec. 3.3, "Boundary and positional handling") ----------------
+# The model's keys carry RoPE: pair k = (dims 2k, 2k+1) read as the complex number
+# x + iy is multiplied by exp(i * position * theta^(-2k/d)), d = 2P real dims in the
+# temporal band (Su et al., RoFormer, Eq. 13-15).  These tests build such keys with
+# numpy complex arithmetic, independently of the oracle's own rotation code.
+
+def _rope(X, position, pairs, theta):
+    """Apply RoPE at `position` to the first `pairs` complex pairs of the last axis of X."""
+    X = np.array(X, dtype=np.float64, copy=True)
+    k = np.arange(pairs)
+    z = X[..., 0:2 * pairs:2] + 1j * X[..., 1:2 * pairs:2]
+    z = z * np.exp(1j * position * theta ** (-2.0 * k / (2 * pairs)))
+    X[..., 0:2 * pairs:2] = z.real
+    X[..., 1:2 * pairs:2] = z.imag
+    return X
+
+
+def test_rope_stored_keys_are_phase_free():
+    """A key the model rotated to its frame's position t is stored exactly as the
+    unrotated key, whatever t; dims outside the temporal band and values are untouched."""
+    rng = np.random.default_rng(41)
+    N, H, D, P, theta = 3, 2, 16, 5, 10000.0
+    mem = OracleMemory(8, 0.3, elems=N * H * D)
+    mem.set_rope(P, theta, N, H, D)
+    raw = []
+    for t in range(6):
+        k0, v = rng.standard_normal((N, H, D)), rng.standard_normal((N, H, D))
+        raw.append((k0, v))
+        mem.insert(_rope(k0, t, P, theta), v)
+    for i, (k0, v) in enumerate(raw):
+        K, V = mem.entry_kv(i)
+        np.testing.assert_allclose(K.reshape(N, H, D), k0, rtol=0, atol=1e-12)
+        np.testing.assert_array_equal(V.reshape(N, H, D), v)
+
+
+def test_rope_without_merges_restores_true_positions():
+    """Budget >= history: re-indexing puts entry i at position t_next - count + i = i,
+    its own frame, so attention over the memory equals attention over the model's own
+    RoPE keys (plain attention, pinned above against numpy)."""
+    rng = np.random.default_rng(42)
+    N, H, D, P, theta, F = 4, 2, 16, 6, 500.0, 5
+    mem = OracleMemory(8, 0.3, elems=N * H * D)
+    mem.set_rope(P, theta, N, H, D)
+    keys, vals = [], []
+    for t in range(F):
+        k = _rope(rng.standard_normal((N, H, D)), t, P, theta)
+        v = rng.standard_normal((N, H, D))
+        keys.append(k)
+        vals.append(v)
+        mem.insert(k, v)
+    Q = _rope(rng.standard_normal((7, H, D)), F, P, theta)
+    out = mem.attend(Q, N, H, D)
+    ref = _numpy_attention(Q, np.concatenate(keys), np.concatenate(vals), 1 / math.sqrt(D))
+    np.testing.assert_allclose(out, ref, rtol=1e-11, atol=1e-12)
+    Kc = _rope(rng.standard_normal((3, H, D)), F, P, theta)
+    Vc = rng.standard_normal((3, H, D))
+    out = mem.attend_ext(Q, Kc, Vc, N, H, D)
+    ref = _numpy_attention(Q, np.concatenate(keys + [Kc]), np.concatenate(vals + [Vc]), 1 / math.sqrt(D))
+    np.testing.assert_allclose(out, ref, rtol=1e-11, atol=1e-12)
+
+
+def test_rope_reindex_after_eviction():
+    """Budget 2 with the anchor: every pass merges the anchor pair and keeps frame 0's
+    block (Algorithm S1), so after frames 0..3 the memory is [frame 0, frame 3].  Re-indexed
+    to positions 2 and 3 (right before the query chunk at 4), the attention keys are frame
+    0's raw key at position 2 and frame 3's at its own position 3."""
+    rng = np.random.default_rng(43)
+    N, H, D, P, theta = 2, 1, 8, 3, 100.0
+    mem = OracleMemory(2, 0.5, anchor=True, elems=N * H * D)
+    mem.set_rope(P, theta, N, H, D)
+    raw = [(rng.standard_normal((N, H, D)), rng.standard_normal((N, H, D))) for _ in range(4)]
+    for t, (k0, v) in enumerate(raw):
+        mem.insert(_rope(k0, t, P, theta), v)
+    slot, first, span, mu = mem.entries()
+    assert list(first) == [0, 3] and list(span) == [3, 1]
+    Q = _rope(rng.standard_normal((5, H, D)), 4, P, theta)
+    out = mem.attend(Q, N, H, D)
+    Kref = np.concatenate([_rope(raw[0][0], 2, P, theta), _rope(raw[3][0], 3, P, theta)])
+    Vref = np.concatenate([raw[0][1], raw[3][1]])
+    np.testing.assert_allclose(out, _numpy_attention(Q, Kref, Vref, 1 / math.sqrt(D)), rtol=1e-11, atol=1e-12)
+    # A wrong direction or offset is caught: position 1 for frame 0 gives other outputs.
+    Kbad = np.concatenate([_rope(raw[0][0], 1, P, theta), _rope(raw[3][0], 3, P, theta)])
+    assert np.max(np.abs(out - _numpy_attention(Q, Kbad, Vref, 1 / math.sqrt(D)))) > 1e-6
+
+
+def test_rope_rejects_bad_arguments():
+    mem = OracleMemory(4, 0.3, elems=2 * 1 * 8)
+    for bad in ((0, 1e4, 2, 1, 8), (5, 1e4, 2, 1, 8), (2, 1.0, 2, 1, 8), (2, 1e4, 3, 1, 8)):
+        with pytest.raises(ValueError):
+            mem.set_rope(*bad)
+    mem.insert(np.zeros(16), np.zeros(16))
+    with pytest.raises(ValueError):
+        mem.set_rope(2, 1e4, 2, 1, 8)
