@@ -317,12 +317,55 @@ def run_cuda(args):
                 "api": "fademem_step_host (pinned host K, V, Q in; out back to pinned host memory), "
                        "timed as one region over the steps"},
     }
+    if args.rope_pairs > 0:
+        line["rope"] = _measure_rope(args, sets, out, flush_l2, stream, dev, cons_ms, hbm_peak)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_queries)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()
+
+
+def _measure_rope(args, sets, out, flush_l2, stream, dev, cons_ms_plain, hbm_peak):
+    """The same workload with temporal RoPE handling on (Sec. 3.3, "Boundary and positional
+    handling"; Wan2.1's temporal band of 22 complex pairs): per step the consolidation call
+    now also runs the re-phase kernel, which writes the re-indexed attention keys of every
+    entry (read stored K + write K_att: count * N * H * D * 2 bytes each way)."""
+    from paper_2606_10671_gb300 import FadeMem
+    mem = FadeMem(M, H, D, N, num_layers=1, beta=BETA, anchor=True, dtype=torch.bfloat16, device=dev,
+                  rope_pairs=args.rope_pairs)
+    for s_ in range(8):
+        K, V, _ = sets[s_ % len(sets)]
+        mem.insert(0, K, V)
+        mem.consolidate()
+    steps = max(20, args.steps // 6)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps + 3):
+        K, V, Q = sets[i % len(sets)]
+        flush_l2()
+        if i >= 3:
+            ev[i - 3][0].record(stream)
+        mem.insert(0, K, V)
+        mem.consolidate()
+        if i >= 3:
+            ev[i - 3][1].record(stream)
+        mem.attend(0, Q, out)
+        if i >= 3:
+            ev[i - 3][2].record(stream)
+    torch.cuda.synchronize()
+    mem.device_status()
+    cons = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    attn = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    rephase_bytes = 2 * M * N * H * D * 2
+    re_ms = max(cons - cons_ms_plain, 1e-6)
+    return {"rope_pairs": args.rope_pairs, "steps": steps, "consolidate_ms_per_step": round(cons, 4),
+            "attend_ms_per_step": round(attn, 4), "value": round(LQ / ((cons + attn) / 1e3), 1), "unit": "tokens/s",
+            "rephase_bytes_per_step": rephase_bytes,
+            "rephase_ms_est": round(re_ms, 4),
+            "rephase_frac_est": round(rephase_bytes / (re_ms / 1e3) / 1e9 / hbm_peak, 4),
+            "note": "rephase time estimated as this consolidate time minus the RoPE-off one; its own ncu "
+                    "duration is in profiles/"}
 
 
 class OracleStep:
@@ -411,6 +454,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--rope-pairs", type=int, default=22,
+                    help="also time the workload with temporal RoPE handling on this many pairs (0: skip)")
     ap.add_argument("--cpu-queries", type=int, default=2340, help="query rows of the cpu_baseline sample")
     ap.add_argument("--ref-queries", type=int, default=240, help="query rows per --impl reference step")
     args = ap.parse_args()

@@ -84,13 +84,27 @@ typedef struct fademem_config {
     int merge_op;          /* fademem_merge_op */
     int dtype;             /* fademem_dtype of K, V, Q, out and the stored memory */
     float scale;           /* softmax scale of q.k; 0 selects 1/sqrt(D) */
+    /* Temporal RoPE handling (Sec. 3.3, "Boundary and positional handling"):
+     * rope_pairs = P complex pairs (dims 2k, 2k+1, k < P) of each head's key
+     * carry the temporal rotary phase, frequencies omega_k = theta^(-k/P).
+     * 0 turns it off (keys are stored and attended as given).  With P > 0,
+     * inserted keys carry their frame's phase (position t = the frame's index)
+     * and are stored with it removed; consolidate then writes the keys
+     * attention uses: entry i of count (temporal order) rotated to position
+     * t_next - count + i, consecutive positions ending right before the next
+     * frame t_next, so the exposed range is bounded by M (the paper does not
+     * give the re-index rule; this is the library's reading).  Queries and the
+     * chunk keys of fademem_attend_ext keep the positions the caller gave. */
+    int rope_pairs;        /* 0 <= P <= head_dim / 2 */
+    double rope_theta;     /* RoPE base; 0 selects 10000 */
 } fademem_config;
 
 typedef struct fademem_ctx *fademem_t;
 
 /* Bytes of device workspace a handle with this configuration needs (the
- * memory of every layer, [L][K|V][H][M][N][D] in the storage dtype, plus
- * metadata and the merge plan), or 0 if the configuration is invalid.
+ * memory of every layer, [L][K|V][H][M][N][D] in the storage dtype -- with
+ * temporal RoPE, [L][K|V|K_attention][H][M][N][D] -- plus metadata and the
+ * merge plan), or 0 if the configuration is invalid.
  * Host only; no CUDA call. */
 FADEMEM_API size_t fademem_workspace_bytes(const fademem_config *cfg);
 

@@ -17,11 +17,11 @@ _OPS = {"weighted": capi.FADEMEM_MERGE_WEIGHTED, "average": capi.FADEMEM_MERGE_A
 
 
 def make_config(budget, heads, head_dim, tokens_per_frame, num_layers=1, beta=0.3, anchor=True, merge_op="weighted",
-                dtype=torch.bfloat16, scale=0.0) -> capi.fademem_config:
+                dtype=torch.bfloat16, scale=0.0, rope_pairs=0, rope_theta=0.0) -> capi.fademem_config:
     return capi.fademem_config(budget=int(budget), heads=int(heads), head_dim=int(head_dim),
                                tokens_per_frame=int(tokens_per_frame), num_layers=int(num_layers), beta=float(beta),
                                anchor=int(bool(anchor)), merge_op=_OPS[merge_op], dtype=_DTYPES[dtype],
-                               scale=float(scale))
+                               scale=float(scale), rope_pairs=int(rope_pairs), rope_theta=float(rope_theta))
 
 
 def _stream_handle(stream) -> int:
@@ -38,9 +38,9 @@ class FadeMem:
     """
 
     def __init__(self, budget, heads, head_dim, tokens_per_frame, num_layers=1, beta=0.3, anchor=True,
-                 merge_op="weighted", dtype=torch.bfloat16, scale=0.0, device="cuda"):
+                 merge_op="weighted", dtype=torch.bfloat16, scale=0.0, device="cuda", rope_pairs=0, rope_theta=0.0):
         self.cfg = make_config(budget, heads, head_dim, tokens_per_frame, num_layers, beta, anchor, merge_op, dtype,
-                               scale)
+                               scale, rope_pairs, rope_theta)
         self.dtype = dtype
         self.device = torch.device(device)
         nbytes = capi.fademem_workspace_bytes(self.cfg)

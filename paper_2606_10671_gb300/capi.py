@@ -43,7 +43,7 @@ class fademem_config(ctypes.Structure):
     _fields_ = [("budget", ctypes.c_int), ("heads", ctypes.c_int), ("head_dim", ctypes.c_int),
                 ("tokens_per_frame", ctypes.c_int), ("num_layers", ctypes.c_int), ("beta", ctypes.c_double),
                 ("anchor", ctypes.c_int), ("merge_op", ctypes.c_int), ("dtype", ctypes.c_int),
-                ("scale", ctypes.c_float)]
+                ("scale", ctypes.c_float), ("rope_pairs", ctypes.c_int), ("rope_theta", ctypes.c_double)]
 
 
 class FadeMemError(RuntimeError):

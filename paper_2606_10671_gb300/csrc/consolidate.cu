@@ -337,8 +337,40 @@ struct ConsolidateArgs {
   int la_frames, la_expected, la_anchor, la_op;
   double la_beta;
   int bx;                 // blocks per (layer, K|V, head) row
+  // Temporal RoPE: K frame sources of the pass are rotated by -(t0 + f) omega_k
+  // on their first rope_pairs complex pairs as they are loaded.
+  int rope_pairs;
+  long long rope_t0;
+  double rope_omega[kMaxRopePairs];
   PassSources srcs;
 };
+
+// (cos a, sin a) of a = position * omega in fp32, with the angle reduced to
+// [-pi, pi] in fp64 first: positions reach tens of thousands of frames, far
+// beyond where an fp32 angle keeps its precision.
+__device__ __forceinline__ float2 rope_cos_sin(double position, double omega) {
+  const double two_pi = 6.283185307179586476925;
+  double ang = position * omega;
+  ang -= two_pi * rint(ang / two_pi);
+  float sn, cs;
+  sincosf((float)ang, &sn, &cs);
+  return make_float2(cs, sn);
+}
+
+// Rotate the complex pairs of one 16-byte vector (x[2e], x[2e+1]; pair index
+// pair0 + e) that lie in the temporal band (pair < P), by the table cs[pair].
+template <int kN>
+__device__ __forceinline__ void rope_rotate_vec(float* x, int pair0, int P, const float2* cs) {
+#pragma unroll
+  for (int e = 0; e < kN / 2; ++e) {
+    if (pair0 + e < P) {
+      const float2 r = cs[pair0 + e];
+      const float x0 = x[2 * e], x1 = x[2 * e + 1];
+      x[2 * e] = x0 * r.x - x1 * r.y;
+      x[2 * e + 1] = x0 * r.y + x1 * r.x;
+    }
+  }
+}
 
 // K2 geometry: one wave of 256-thread blocks, 4 per SM (64 registers a
 // thread), spread over the (layer, K|V, head) rows.  Each thread owns one
@@ -350,11 +382,12 @@ struct ConsolidateArgs {
 // which touch at most 2F entries, plus F frame copies, so kNS = 3F suffices;
 // a larger plan is refused through the status word.
 constexpr int kConsThreads = 256;
-// Resident blocks per SM: 4 (64 registers) while the sources fit, 3 for 12.
-__host__ __device__ constexpr int cons_blocks_per_sm(int ns_max) { return ns_max <= 9 ? 4 : 3; }
+// Resident blocks per SM: 4 (64 registers) while the sources fit, 3 for 12
+// sources or with the RoPE rotation.
+__host__ __device__ constexpr int cons_blocks_per_sm(int ns_max, bool rope) { return ns_max <= 9 && !rope ? 4 : 3; }
 
-template <typename T, bool kMax, int kNS>
-__global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consolidate_kernel(
+template <typename T, bool kMax, int kNS, bool kRope>
+__global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS, kRope)) consolidate_kernel(
     const __grid_constant__ ConsolidateArgs a) {
   using V = Vec<T>;
   __shared__ const T* s_base[kMaxSrc];  // source k at token n: s_base[k] + n * (token stride) + d
@@ -362,6 +395,8 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consoli
   __shared__ float s_w[kMaxSrc];
   __shared__ unsigned s_frame_mask, s_end_mask;  // bit k: source k is a frame / ends its run
   __shared__ int s_ns;
+  __shared__ int s_frame_of[kMaxSrc];                      // frame index f of a frame source
+  __shared__ float2 s_rope_cs[kRope ? kMaxPassFrames : 1][kRope ? kMaxRopePairs : 1];  // by -(t0 + f) omega_k
   // Launched as a programmatic dependent of the schedule kernel: wait for it
   // (and every earlier grid of the stream) before reading any global memory.
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -406,6 +441,7 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consoli
                         : cache + (size_t)r * a.slab_elems;
       s_w[k] = p.src_w[k];
       s_dst[k] = cache + (size_t)(bad ? 0 : p.dest_slot[dk]) * a.slab_elems;
+      s_frame_of[k] = frame ? -r - 1 : 0;
     }
     const unsigned fm = __ballot_sync(0xffffffffu, frame), em = __ballot_sync(0xffffffffu, end);
     if (__any_sync(0xffffffffu, bad)) ns = kMaxSrc + 1;
@@ -417,6 +453,14 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consoli
         atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
         atomicAdd(&a.totals[1], 1ull);
       }
+    }
+  }
+  // Temporal RoPE: the K rows of this pass's frames lose their phase.
+  const bool rope = kRope && kv == 0;
+  if (kRope && rope) {
+    for (int t = threadIdx.x; t < kMaxPassFrames * a.rope_pairs; t += blockDim.x) {
+      const int f = t / a.rope_pairs, k = t % a.rope_pairs;
+      s_rope_cs[f][k] = rope_cos_sin(-(double)(a.rope_t0 + f), a.rope_omega[k]);
     }
   }
   __syncthreads();
@@ -450,6 +494,8 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS)) consoli
       if (k < ns) {
         float x[V::kN];
         V::unpack(raw[k], x);
+        if (kRope && rope && ((fmask >> k) & 1) && (int)d < 2 * a.rope_pairs)
+          rope_rotate_vec<V::kN>(x, (int)d / 2, a.rope_pairs, s_rope_cs[s_frame_of[k]]);
         const float w = s_w[k];
 #pragma unroll
         for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? fmaxf(acc[e], x[e]) : fmaf(w, x[e], acc[e]);
@@ -473,7 +519,8 @@ cudaError_t launch_schedule(const DevState* in, DevState* out, unsigned int* sta
 }
 
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
-                               int frames, int op, const Lookahead& la, cudaStream_t stream) {
+                               int frames, int op, const Lookahead& la, const PassRope& rope,
+                               cudaStream_t stream) {
   static_assert(kMaxSrc == 3 * kMaxPassFrames, "a pass of F frames has at most 3F sources");
   ConsolidateArgs a;
   a.la_in = la.in;
@@ -485,6 +532,9 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   a.la_anchor = la.anchor;
   a.la_op = la.op;
   a.la_beta = la.beta;
+  a.rope_pairs = rope.pairs;
+  a.rope_t0 = rope.t0;
+  for (int k = 0; k < kMaxRopePairs; ++k) a.rope_omega[k] = rope.omega[k];
   a.cache = reinterpret_cast<char*>(cache_base);
   a.st = st;
   a.L = g.L; a.H = g.H; a.M = g.M; a.N = g.N; a.D = g.D;
@@ -508,7 +558,7 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   }
   const int nsb = frames <= 2 ? 0 : frames == 3 ? 1 : 2;  // sources <= 3F: 6, 9 or 12
   const int rows = g.L * 2 * g.H;
-  int bx = (num_sms * cons_blocks_per_sm(6 + 3 * nsb) - 1) / rows;  // - 1: the lookahead block
+  int bx = (num_sms * cons_blocks_per_sm(6 + 3 * nsb, rope.pairs > 0) - 1) / rows;  // - 1: the lookahead block
   const int bx_max = (nvec + kConsThreads - 1) / kConsThreads;
   if (bx > bx_max) bx = bx_max;
   if (bx < 1) bx = 1;
@@ -516,15 +566,14 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   dim3 grid(1 + bx * rows);  // block 0: the lookahead schedule
   const bool mx = op == FADEMEM_MERGE_MAX_POOL;
   using Kern = void (*)(const ConsolidateArgs);
-  static const Kern kerns[2][2][3] = {
-      {{consolidate_kernel<float, false, 6>, consolidate_kernel<float, false, 9>,
-        consolidate_kernel<float, false, 12>},
-       {consolidate_kernel<float, true, 6>, consolidate_kernel<float, true, 9>, consolidate_kernel<float, true, 12>}},
-      {{consolidate_kernel<__nv_bfloat16, false, 6>, consolidate_kernel<__nv_bfloat16, false, 9>,
-        consolidate_kernel<__nv_bfloat16, false, 12>},
-       {consolidate_kernel<__nv_bfloat16, true, 6>, consolidate_kernel<__nv_bfloat16, true, 9>,
-        consolidate_kernel<__nv_bfloat16, true, 12>}}};
-  const Kern kern = kerns[g.dtype == FADEMEM_BF16 ? 1 : 0][mx ? 1 : 0][nsb];
+#define FM_K2(T, MX, R) {consolidate_kernel<T, MX, 6, R>, consolidate_kernel<T, MX, 9, R>, consolidate_kernel<T, MX, 12, R>}
+  static const Kern kerns[2][2][2][3] = {
+      {{FM_K2(float, false, false), FM_K2(float, true, false)},
+       {FM_K2(__nv_bfloat16, false, false), FM_K2(__nv_bfloat16, true, false)}},
+      {{FM_K2(float, false, true), FM_K2(float, true, true)},
+       {FM_K2(__nv_bfloat16, false, true), FM_K2(__nv_bfloat16, true, true)}}};
+#undef FM_K2
+  const Kern kern = kerns[rope.pairs > 0 ? 1 : 0][g.dtype == FADEMEM_BF16 ? 1 : 0][mx ? 1 : 0][nsb];
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = dim3(kConsThreads);
@@ -536,6 +585,112 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, a);
+}
+
+
+// ---- K2b: temporal RoPE re-index ------------------------------------------
+
+namespace {
+
+struct RephaseArgs {
+  char* cache;
+  const DevState* st;
+  int H, M, N, D, count, bx, dv_shift, pairs;
+  long long t_next;
+  size_t slab_elems, kv_elems, layer_elems;
+  double omega[kMaxRopePairs];
+};
+
+// One wave of 256-thread blocks over the (layer, head, entry) rows; block x of
+// a row streams 16-byte vectors of the entry's stored K slab to the same place
+// in the K_att block, rotating the vectors of the temporal band.  Four loads
+// are in flight per thread.  HBM-bound: count * N * D * elem read and written
+// per (layer, head).
+template <typename T>
+__global__ void __launch_bounds__(256) rephase_kernel(const __grid_constant__ RephaseArgs a) {
+  using V = Vec<T>;
+  __shared__ float2 s_cs[kMaxRopePairs];
+  const int bx = (int)blockIdx.x % a.bx;
+  const int row = (int)blockIdx.x / a.bx;
+  const int i = row % a.count;
+  const int h = (row / a.count) % a.H;
+  const int l = row / (a.count * a.H);
+  int slot = a.st->meta.slot[i];
+  if (slot < 0 || slot >= a.M) return;  // not a valid table (refused earlier by the schedule checks)
+  const double tau = (double)(a.t_next - a.count + i);  // re-indexed position of entry i
+  for (int k = threadIdx.x; k < a.pairs; k += blockDim.x) s_cs[k] = rope_cos_sin(tau, a.omega[k]);
+  __syncthreads();
+  const T* src = reinterpret_cast<const T*>(a.cache) + (size_t)l * a.layer_elems + (size_t)h * a.M * a.slab_elems +
+                 (size_t)slot * a.slab_elems;
+  T* dst = const_cast<T*>(src) + 2 * a.kv_elems;  // K_att follows K and V
+  const int nvec = a.N << a.dv_shift;
+  const int dvmask = (1 << a.dv_shift) - 1;
+  const int step = a.bx * blockDim.x;
+  constexpr int kU = 4;
+  for (int v0 = bx * blockDim.x + threadIdx.x; v0 < nvec; v0 += kU * step) {
+    uint4 raw[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int v = v0 + u * step;
+      if (v < nvec) raw[u] = __ldcs(reinterpret_cast<const uint4*>(src) + v);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int v = v0 + u * step;
+      if (v >= nvec) continue;
+      const int d = (v & dvmask) * V::kN;
+      uint4 w = raw[u];
+      if (d < 2 * a.pairs) {
+        float x[V::kN];
+        V::unpack(w, x);
+        rope_rotate_vec<V::kN>(x, d / 2, a.pairs, s_cs);
+        w = V::pack(x);
+      }
+      reinterpret_cast<uint4*>(dst)[v] = w;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* st, int count, long long t_next,
+                           cudaStream_t stream) {
+  if (count <= 0 || g.rope_pairs <= 0) return cudaSuccess;
+  RephaseArgs a;
+  a.cache = reinterpret_cast<char*>(cache_base);
+  a.st = st;
+  a.H = g.H; a.M = g.M; a.N = g.N; a.D = g.D;
+  a.count = count;
+  a.pairs = g.rope_pairs;
+  a.t_next = t_next;
+  a.slab_elems = g.slab_elems;
+  a.kv_elems = g.kv_elems;
+  a.layer_elems = g.layer_bytes / g.elem;
+  for (int k = 0; k < kMaxRopePairs; ++k) a.omega[k] = g.rope_omega[k];
+  const int per_vec = g.dtype == FADEMEM_BF16 ? 8 : 4;
+  int dv = g.D / per_vec, shift = 0;
+  while ((1 << shift) < dv) ++shift;
+  a.dv_shift = shift;
+  static int num_sms = 0;
+  if (num_sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                   cudaSuccess)
+      num_sms = 148;
+  }
+  const long long rows = (long long)g.L * g.H * count;
+  const int nvec = g.N * dv;
+  long long bx = (long long)num_sms * 8 / rows;  // one wave of 8 resident blocks per SM
+  const long long bx_max = (nvec + 255) / 256;
+  if (bx > bx_max) bx = bx_max;
+  if (bx < 1) bx = 1;
+  a.bx = (int)bx;
+  const dim3 grid((unsigned)(bx * rows));
+  if (g.dtype == FADEMEM_BF16)
+    rephase_kernel<__nv_bfloat16><<<grid, 256, 0, stream>>>(a);
+  else
+    rephase_kernel<float><<<grid, 256, 0, stream>>>(a);
+  return cudaGetLastError();
 }
 
 }  // namespace fademem

@@ -95,6 +95,10 @@ static fademem_status check_config(const fademem_config* c, Geometry* g) {
   if (lk > (1LL << 30)) return fail(FADEMEM_ERR_INVALID_ARG, "budget * tokens_per_frame too large");
   if ((long long)c->tokens_per_frame * c->heads * c->head_dim >= (1LL << 31))
     return fail(FADEMEM_ERR_INVALID_ARG, "tokens_per_frame * heads * head_dim must be below 2^31");
+  if (c->rope_pairs < 0 || 2 * c->rope_pairs > c->head_dim)
+    return fail(FADEMEM_ERR_INVALID_ARG, "rope_pairs must be in [0, head_dim / 2] (got %d)", c->rope_pairs);
+  if (c->rope_pairs > 0 && !(c->rope_theta == 0.0 || (c->rope_theta > 1.0 && c->rope_theta < 1e30)))
+    return fail(FADEMEM_ERR_INVALID_ARG, "rope_theta must be 0 (10000) or above 1");
   if (g) {
     g->L = c->num_layers;
     g->H = c->heads;
@@ -106,7 +110,11 @@ static fademem_status check_config(const fademem_config* c, Geometry* g) {
     g->slab_elems = (size_t)g->N * g->D;
     g->kv_elems = (size_t)g->H * g->M * g->slab_elems;
     g->state_bytes = 256 + 2 * round_up(sizeof(DevState), 256);
-    g->layer_bytes = round_up(2 * g->kv_elems * g->elem, 256);
+    g->layer_bytes = round_up((c->rope_pairs > 0 ? 3 : 2) * g->kv_elems * g->elem, 256);
+    g->rope_pairs = c->rope_pairs;
+    const double theta = c->rope_theta == 0.0 ? 10000.0 : c->rope_theta;
+    for (int k = 0; k < kMaxRopePairs; ++k)
+      g->rope_omega[k] = k < c->rope_pairs ? pow(theta, -(double)k / (double)c->rope_pairs) : 0.0;
     g->total_bytes = g->state_bytes + (size_t)g->L * g->layer_bytes;
   }
   return FADEMEM_OK;
@@ -254,7 +262,11 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
     la.anchor = h->cfg.anchor;
     la.op = h->cfg.merge_op;
     la.beta = h->cfg.beta;
-    e = launch_consolidate(h->g, h->cache, cur_state(h), srcs, nf, h->cfg.merge_op, la, stream);
+    PassRope rope;
+    rope.pairs = h->g.rope_pairs;
+    rope.t0 = h->frames;
+    memcpy(rope.omega, h->g.rope_omega, sizeof(rope.omega));
+    e = launch_consolidate(h->g, h->cache, cur_state(h), srcs, nf, h->cfg.merge_op, la, rope, stream);
     if (e != cudaSuccess) return cuda_fail(e, "launching the consolidation kernel");
     ++h->launches;
     h->frames = frames_after;
@@ -270,6 +282,12 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   for (int l = 0; l < L; ++l) {
     h->pending[l].clear();
     h->pending_frames[l] = 0;
+  }
+  if (h->g.rope_pairs > 0) {
+    // Keys for attention: every entry rotated to its re-indexed position.
+    cudaError_t e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the re-phase kernel");
+    ++h->launches;
   }
   if (make_la) {
     h->la_valid = true;
@@ -295,8 +313,10 @@ static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const v
   if (h->count == 0 && ncur == 0) return fail(FADEMEM_ERR_EMPTY, "the memory holds no entries");
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   const int Lk = h->count * h->g.N;
-  const char* Kc = h->cache + (size_t)layer * h->g.layer_bytes;
-  const char* Vc = Kc + h->g.kv_elems * h->g.elem;
+  const char* Kmem = h->cache + (size_t)layer * h->g.layer_bytes;
+  const char* Vc = Kmem + h->g.kv_elems * h->g.elem;
+  // With temporal RoPE, attention reads the re-indexed keys (after V).
+  const char* Kc = h->g.rope_pairs > 0 ? Vc + h->g.kv_elems * h->g.elem : Kmem;
   cudaError_t e;
   if (h->g.dtype == FADEMEM_F32) {
     e = launch_attend_f32(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, reinterpret_cast<const float*>(Q),

@@ -15,6 +15,7 @@ constexpr int kMaxPassFrames = 4;
 constexpr int kMaxDest = 2 * kMaxPassFrames;
 constexpr int kMaxSrc = 3 * kMaxPassFrames;
 constexpr int kMaxEntries = FADEMEM_MAX_BUDGET + 1;
+constexpr int kMaxRopePairs = 64;  // head_dim / 2 at head_dim 128
 
 // Device status word bits (fademem_get_device_status).
 constexpr uint32_t kStatusTimeout = 1u << 0;      // a bounded mbarrier wait gave up
@@ -54,7 +55,8 @@ struct DevState {
   DevPlan plan;
 };
 
-// Layout of one layer in the workspace: K then V, each [H][M][N][D].
+// Layout of one layer in the workspace: K then V, each [H][M][N][D], then
+// (temporal RoPE only) the attention keys K_att [H][M][N][D].
 struct Geometry {
   int L, H, M, N, D;
   int dtype;             // fademem_dtype
@@ -62,8 +64,10 @@ struct Geometry {
   size_t slab_elems;     // N * D
   size_t kv_elems;       // H * M * N * D (one of K or V of one layer)
   size_t state_bytes;    // status word + two DevState buffers, each rounded to 256
-  size_t layer_bytes;    // 2 * kv_elems * elem, rounded to 256
+  size_t layer_bytes;    // (2 or 3) * kv_elems * elem, rounded to 256
   size_t total_bytes;
+  int rope_pairs;        // temporal RoPE pairs P (0: off)
+  double rope_omega[kMaxRopePairs];  // omega_k = theta^(-k/P)
 };
 
 // Per-pass source pointers: layer l's K (or V) frames of the pass start at
@@ -80,6 +84,15 @@ cudaError_t launch_schedule(const DevState* in, DevState* out, unsigned int* sta
                             int anchor, int op, int expected_count, cudaStream_t stream);
 // Schedule of the next pass computed inside the consolidation kernel (by one
 // extra block) from the entry table `in` into `out`; out == nullptr skips it.
+// Temporal RoPE of one consolidation pass: frame f of the pass sits at
+// position t0 + f; K frame sources are rotated by -(t0 + f) omega_k as they
+// are loaded (stored keys carry no phase).
+struct PassRope {
+  int pairs;             // 0: no rotation
+  long long t0;
+  double omega[kMaxRopePairs];
+};
+
 struct Lookahead {
   const DevState* in;
   DevState* out;
@@ -89,7 +102,12 @@ struct Lookahead {
   double beta;
 };
 cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevState* st, const PassSources& srcs,
-                               int frames, int op, const Lookahead& la, cudaStream_t stream);
+                               int frames, int op, const Lookahead& la, const PassRope& rope, cudaStream_t stream);
+// Temporal RoPE re-index: for every layer, head and entry i < count of st's
+// entry table, K_att[slot_i] = stored K[slot_i] rotated to position
+// t_next - count + i (the rest of each row copied unchanged).
+cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* st, int count, long long t_next,
+                           cudaStream_t stream);
 // Attention over Lk memory keys (Kc/Vc: one layer's [H][M][N][D] memory) followed
 // by Lk2 current-chunk keys (Kcur/Vcur: [Lk2][H][D]); either count may be 0.
 cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,

@@ -49,16 +49,20 @@ class Pair:
 
     def __init__(self, budget, heads, head_dim, tokens, beta=0.3, anchor=True, op="weighted",
                  dtype=torch.bfloat16, layers=1, seed=0, rho=rho_const(0.9), tracked_heads=None, device_gen=False,
-                 oracle_layers=None):
+                 oracle_layers=None, rope_pairs=0, rope_theta=10000.0):
         from paper_2606_10671_gb300 import FadeMem
         self.M, self.H, self.D, self.N, self.L = budget, heads, head_dim, tokens, layers
         self.dtype = dtype
         self.tracked = list(range(heads)) if tracked_heads is None else list(tracked_heads)
         self.gpu = FadeMem(budget, heads, head_dim, tokens, num_layers=layers, beta=beta, anchor=anchor, merge_op=op,
-                           dtype=dtype)
+                           dtype=dtype, rope_pairs=rope_pairs, rope_theta=rope_theta)
+        self.rope = rope_pairs > 0
         elems = tokens * len(self.tracked) * head_dim
         self.ora_layers = list(range(layers)) if oracle_layers is None else list(oracle_layers)
         self.ora = {l: OracleMemory(budget, beta, anchor=anchor, op=OPS[op], elems=elems) for l in self.ora_layers}
+        if rope_pairs:
+            for o in self.ora.values():
+                o.set_rope(rope_pairs, rope_theta, tokens, len(self.tracked), head_dim)
         shape = (tokens, heads, head_dim)
         if device_gen:
             self.gens = [(DeviceAR1(shape, seed, KIND_K, l, rho, dtype), DeviceAR1(shape, seed, KIND_V, l, rho, dtype))
@@ -159,12 +163,18 @@ class Pair:
             r = self.rounds.get((int(first[i]), int(span[i])), 0)
             for got, ref, nm in ((kg, Ko, "K"), (vg, Vo, "V")):
                 err = np.abs(got - ref)
-                bound = r * (BF16_U + 2.0 ** -20) * self.input_max + 1e-12  # + fp32 accumulation
+                # Temporal RoPE: a stored K block is rotated before its rounding, so even a
+                # copy is rounded once, and rotated components reach sqrt(2) * A.  (The
+                # anchor's frame 0 rotates by 0 and stays exact, within this bound.)
+                rk, amax = (max(r, 1), np.sqrt(2.0) * self.input_max) if self.rope and nm == "K" \
+                    else (r, self.input_max)
+                bound = rk * (BF16_U + 2.0 ** -20) * amax + 1e-12  # + fp32 accumulation
+                r_rms = rk
                 assert np.all(np.isfinite(got)), nm
                 assert err.max() <= bound, f"{nm} entry {i} slot {s}: max|diff| {err.max():.3e} > {bound:.3e} (r={r})"
                 rms = np.sqrt(np.mean(err ** 2))
-                assert rms <= 2 * np.sqrt(r) * BF16_U * np.sqrt(np.mean(ref ** 2)) + 1e-12, \
-                    f"{nm} entry {i} slot {s}: rms diff {rms:.3e} (r={r})"
+                assert rms <= 2 * np.sqrt(r_rms) * BF16_U * np.sqrt(np.mean(ref ** 2)) + 1e-12, \
+                    f"{nm} entry {i} slot {s}: rms diff {rms:.3e} (r={r_rms})"
                 worst = max(worst, float(err.max()))
         return worst
 

@@ -52,8 +52,13 @@ def test_workspace_bytes(cuda_lib):
     n32 = capi.fademem_workspace_bytes(_cfg(dtype=torch.float32))
     assert n32 - n == kv
     for bad in (dict(budget=1), dict(budget=65), dict(heads=0), dict(head_dim=96), dict(tokens_per_frame=0),
-                dict(num_layers=0), dict(num_layers=129), dict(beta=0.0), dict(beta=1.5), dict(head_dim=64)):
+                dict(num_layers=0), dict(num_layers=129), dict(beta=0.0), dict(beta=1.5), dict(head_dim=64),
+                dict(rope_pairs=-1), dict(rope_pairs=65), dict(rope_pairs=4, rope_theta=0.5)):
         assert capi.fademem_workspace_bytes(_cfg(**bad)) == 0, bad
+    # Temporal RoPE adds the attention keys: a third [H][M][N][D] block per layer.
+    nr = capi.fademem_workspace_bytes(_cfg(rope_pairs=22))
+    assert nr - n == kv // 2 + (-(kv + kv // 2) % 256) - (-kv % 256)
+    assert capi.fademem_workspace_bytes(_cfg(rope_pairs=64, rope_theta=500.0)) == nr
 
 
 def _create_status(cfg, ws=FAKE_WS, nbytes=None):

@@ -275,3 +275,46 @@ def test_step_host_matches_device_path():
     assert a.counts() == b.counts() == (M, 6 * F)
     a.device_status()
     b.device_status()
+
+
+@pytest.mark.parametrize("dtype,D,N,M,P", [(torch.float32, 64, 64, 8, 10), (torch.bfloat16, 128, 100, 5, 22)])
+def test_rope_memory_and_attention(dtype, D, N, M, P):
+    """Temporal RoPE (Sec. 3.3, "Boundary and positional handling"): stored keys lose
+    their frame's phase in the consolidation kernel; attention keys are re-indexed to
+    t_next - count + i by the re-phase kernel.  Entries bit-exact, memory and
+    attention (with and without the current chunk) against the oracle."""
+    p = Pair(M, 2, D, N, beta=0.3, dtype=dtype, seed=15, rope_pairs=P, rope_theta=10000.0)
+    for seg in range(9):
+        p.step(3)
+        p.check_entries()
+        p.check_memory()
+        if seg in (0, 1, 4, 8):
+            p.check_attend(p.queries(130, step=seg))
+            Kc, Vc = p.chunk(150, step=seg)
+            p.check_attend_ext(p.queries(130, step=seg + 20), Kc, Vc)
+    p.gpu.device_status()
+
+
+def test_rope_varying_frames_multipass():
+    """RoPE positions across multi-pass calls (frames 5 and 7 split into passes of <= 4),
+    the lookahead schedule and a reset: each pass de-phases its frames at their own index."""
+    p = Pair(6, 2, 64, 8, beta=0.3, dtype=torch.float32, seed=16, rope_pairs=16, rope_theta=500.0)
+    for F in [3, 5, 3, 3, 7, 1, 2, 3]:
+        p.step(F)
+        p.check_entries()
+        p.check_memory()
+        p.check_attend(p.queries(20, step=F))
+    p.gpu.device_status()
+
+
+def test_rope_wan13b_full_size():
+    """Wan-1.3B single layer with Wan's temporal band (22 of 64 pairs), steady state:
+    sampled query rows against the oracle."""
+    p = Pair(21, 12, 128, 1560, beta=0.3, dtype=torch.bfloat16, seed=17, tracked_heads=[0, 11], device_gen=True,
+             rope_pairs=22)
+    for seg in range(9):
+        p.step(3)
+    p.check_entries()
+    rows = np.array([0, 17, 2048, 4095, 4679])
+    p.check_attend(p.queries(4680, step=9), rows=rows)
+    p.gpu.device_status()
