@@ -318,3 +318,20 @@ def test_rope_wan13b_full_size():
     rows = np.array([0, 17, 2048, 4095, 4679])
     p.check_attend(p.queries(4680, step=9), rows=rows)
     p.gpu.device_status()
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("op", ["weighted", "max_pool"])
+@pytest.mark.parametrize("F", [2, 3, 4])
+@pytest.mark.parametrize("rope", [0, 22])
+def test_consolidation_kernel_variants(dtype, op, F, rope):
+    """Every consolidation kernel instance (source bound 3F = 6, 9, 12; linear or max;
+    with and without the RoPE de-phase), in steady state with chained merges."""
+    D = 128
+    p = Pair(6, 2, D, 40, beta=0.3, dtype=dtype, op=op, seed=100 + F + rope, rope_pairs=rope)
+    for seg in range(7):
+        p.step(F)
+        p.check_entries()
+        p.check_memory()
+    p.check_attend(p.queries(50, step=1))
+    p.gpu.device_status()
