@@ -40,6 +40,13 @@ import torch  # noqa: E402
 H, D, N, F, M, BETA = 12, 128, 1560, 3, 21, 0.3
 LQ = F * N
 WORKLOAD = "wan2.1-1.3b-shaped single layer: H=12 D=128 N=1560 frames/segment=3 Lq=4680 M=21 beta=0.3 bf16"
+# --workload: the headline (default) and the per-layer unit of the 14B model (H=40), timed as one
+# attend + one consolidate at that shape.
+WORKLOADS = {
+    "wan1.3b": (12, WORKLOAD),
+    "wan14b": (40, "wan2.1-14b-shaped single layer (one layer of the 40-layer model): H=40 D=128 N=1560 "
+                   "frames/segment=3 Lq=4680 M=21 beta=0.3 bf16"),
+}
 METRIC = "query tokens/s per layer (attend+consolidate)"
 
 
@@ -53,6 +60,8 @@ def _peaks():
 
 
 def _profiled_traffic(profile: str, source: str):
+    if H != 12:
+        return None  # the committed captures are of the default workload
     """DRAM bytes per launch from a committed ncu summary, or None if the kernel
     source changed since those counters were taken (hash recorded in the summary)."""
     import hashlib
@@ -454,6 +463,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="wan1.3b")
     ap.add_argument("--rope-pairs", type=int, default=22,
                     help="also time the workload with temporal RoPE handling on this many pairs (0: skip)")
     ap.add_argument("--cpu-queries", type=int, default=2340, help="query rows of the cpu_baseline sample")
@@ -461,6 +471,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    global H, WORKLOAD
+    H, WORKLOAD = WORKLOADS[args.workload]
     if args.impl == "reference":
         run_reference(args)
     else:
