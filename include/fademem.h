@@ -237,12 +237,13 @@ FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
 FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void *stream);
 
 /* Device staging bytes fademem_step_host needs for segments of `nframes`
- * frames per layer and `Lq` query tokens: two slots of the inputs (K and V
- * of every layer, Q) plus one output block.  0 if cfg is invalid or
- * nframes/Lq out of range.  No CUDA call is made. */
+ * frames per layer and `Lq` query tokens: two slots, each holding the inputs
+ * (K and V of every layer, Q) and the output block of one step.  0 if cfg is
+ * invalid or nframes/Lq out of range.  No CUDA call is made. */
 FADEMEM_API size_t fademem_host_staging_bytes(const fademem_config *cfg, int nframes, int Lq);
 
-/* One step of a serving loop with the inputs and the result in HOST memory:
+/* One step of a serving loop with the inputs and the result in HOST memory
+ * (the paper has no counterpart: it is the library's own serving entry):
  * copy the segment's frames and the queries in, insert the frames on every
  * layer, consolidate (Algorithm S1 and the merges of Sec. 3.3), attend the
  * queries over `layer`'s memory (Sec. 3.3, last paragraph), and copy the
@@ -256,11 +257,14 @@ FADEMEM_API size_t fademem_host_staging_bytes(const fademem_config *cfg, int nfr
  *                         fademem_host_staging_bytes(cfg, nframes, Lq) bytes,
  *                         16-byte aligned, used by this handle only and the
  *                         same on every call with these sizes
- * The host-to-device copies go on a stream of the handle's own and alternate
- * between the two staging slots, so the copies of the next call overlap the
- * work of this one.  Everything else, including the copy of the output to
- * out_host, is enqueued on `stream`: once `stream` has synchronised, out_host
- * holds this call's output and the host inputs of this call may be reused.
+ * The step runs on three streams of the handle's own -- host-to-device
+ * copies, kernels, device-to-host copy -- and alternates between the two
+ * staging slots, so consecutive calls overlap: the next call's input copies
+ * and kernels run while this call's output is copied out.  The step starts
+ * after the work enqueued on `stream` before the call, and `stream` waits for
+ * the step's output copy: once `stream` has synchronised, out_host holds this
+ * call's output and the host inputs of this call may be reused.  Other work
+ * of this handle must be ordered through `stream` as well.
  * Errors as fademem_insert / fademem_consolidate / fademem_attend, plus
  * FADEMEM_ERR_WORKSPACE if staging is too small or misaligned. */
 FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void *const *K_host, const void *const *V_host,

@@ -58,13 +58,22 @@ struct fademem_ctx {
   int la_frames;         // the frame count it assumed
   bool la_enabled;
   unsigned long long launches = 0;  // kernels this handle launched
-  // fademem_step_host: the copy stream, and per staging slot the events "inputs
-  // copied" and "slot no longer read by the compute stream".
-  cudaStream_t copy_stream = nullptr;
+  // fademem_step_host: its own compute, host-to-device and device-to-host
+  // streams, and per staging slot the events "inputs copied in" (ev_in), "step
+  // computed: inputs consumed, output written" (ev_att) and "output copied out"
+  // (ev_out); ev_entry marks the caller's stream at entry.
+  cudaStream_t comp_stream = nullptr, h2d_stream = nullptr, d2h_stream = nullptr;
+  cudaEvent_t ev_entry = nullptr;
   cudaEvent_t ev_in[2] = {nullptr, nullptr};
-  cudaEvent_t ev_done[2] = {nullptr, nullptr};
-  bool done_recorded[2] = {false, false};
+  cudaEvent_t ev_att[2] = {nullptr, nullptr};
+  cudaEvent_t ev_out[2] = {nullptr, nullptr};
+  bool slot_used[2] = {false, false};
   int host_slot = 0;
+  // The handle's last enqueuing call was fademem_step_host on this stream: the
+  // next step needs no wait on the caller's stream (nothing of the handle can
+  // have been enqueued there since).  Every other enqueuing entry point clears it.
+  bool chained = false;
+  cudaStream_t chained_stream = nullptr;
   int count;             // entries, = min(frames, M) (one merge per insert beyond the budget)
   long long frames;      // consolidated frames
   std::vector<Chunk> pending[FADEMEM_MAX_LAYERS];
@@ -181,6 +190,7 @@ static DevState* cur_state(fademem_t h) { return h->st_buf[h->cur]; }
 
 static fademem_status ensure_init(fademem_t h, cudaStream_t stream) {
   if (!h->need_init) return FADEMEM_OK;
+  h->chained = false;
   cudaError_t e = cudaMemsetAsync(h->ws, 0, h->g.state_bytes, stream);
   if (e != cudaSuccess) return cuda_fail(e, "initialising the entry table");
   h->cur = 0;
@@ -192,6 +202,7 @@ static fademem_status ensure_init(fademem_t h, cudaStream_t stream) {
 
 FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->chained = false;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   const int L = h->g.L;
   const int F = h->pending_frames[0];
@@ -299,6 +310,7 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
 static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const void* Kcur, const void* Vcur,
                                   int ncur, void* out, int Lq, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->chained = false;
   if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
   if (!Q || !out) return fail(FADEMEM_ERR_INVALID_ARG, "Q or out is NULL");
   if (!aligned16(Q) || !aligned16(out)) return fail(FADEMEM_ERR_INVALID_ARG, "Q and out must be 16-byte aligned");
@@ -438,6 +450,7 @@ FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void* stream_,
 
 FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->chained = false;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   fademem_status s = ensure_init(h, stream);
   if (s != FADEMEM_OK) return s;
@@ -449,6 +462,7 @@ FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void* stre
 
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->chained = false;
   h->la_valid = false;
   h->need_init = true;
   fademem_status s = ensure_init(h, reinterpret_cast<cudaStream_t>(stream_));
@@ -500,6 +514,7 @@ extern "C" {
 
 FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream_) {
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  h->chained = false;
   if (h->g.M + 1 > kMaxEntries)
     return fail(FADEMEM_ERR_UNSUPPORTED, "budget %d does not fit the %d-byte no-alloc scratch", h->g.M,
                 FADEMEM_NOALLOC_SCRATCH_BYTES);
@@ -528,17 +543,16 @@ FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream
 }
 
 // Staging layout of fademem_step_host: slot s (s = 0, 1) holds, 256-byte
-// aligned, K then V of every layer and then Q; the output block follows both.
+// aligned, K then V of every layer, then Q, then the output block.
 struct HostStaging {
-  size_t frame_bytes, q_bytes, slot_bytes, out_off, total;
+  size_t frame_bytes, q_bytes, slot_bytes, total;
 };
 static bool host_staging(const Geometry& g, int nframes, int Lq, HostStaging* st) {
   if (nframes < 1 || nframes > FADEMEM_MAX_PENDING || Lq < 1 || Lq > (1 << 24)) return false;
   st->frame_bytes = round_up((size_t)nframes * g.N * g.H * g.D * g.elem, 256);
   st->q_bytes = round_up((size_t)Lq * g.H * g.D * g.elem, 256);
-  st->slot_bytes = 2 * (size_t)g.L * st->frame_bytes + st->q_bytes;
-  st->out_off = 2 * st->slot_bytes;
-  st->total = st->out_off + st->q_bytes;
+  st->slot_bytes = 2 * (size_t)g.L * st->frame_bytes + 2 * st->q_bytes;
+  st->total = 2 * st->slot_bytes;
   return true;
 }
 
@@ -565,61 +579,91 @@ FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void* const* K_h
                 staging_bytes, staging);
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   cudaError_t e;
-  if (!h->copy_stream) {
-    e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
-    if (e != cudaSuccess) return cuda_fail(e, "creating the copy stream");
-    for (int s = 0; s < 2; ++s) {
-      if ((e = cudaEventCreateWithFlags(&h->ev_in[s], cudaEventDisableTiming)) != cudaSuccess ||
-          (e = cudaEventCreateWithFlags(&h->ev_done[s], cudaEventDisableTiming)) != cudaSuccess)
-        return cuda_fail(e, "creating the copy events");
-    }
+  if (!h->comp_stream) {
+    cudaStream_t* ss[3] = {&h->comp_stream, &h->h2d_stream, &h->d2h_stream};
+    for (cudaStream_t* x : ss)
+      if ((e = cudaStreamCreateWithFlags(x, cudaStreamNonBlocking)) != cudaSuccess)
+        return cuda_fail(e, "creating the step streams");
+    if ((e = cudaEventCreateWithFlags(&h->ev_entry, cudaEventDisableTiming)) != cudaSuccess)
+      return cuda_fail(e, "creating the step events");
+    for (int k = 0; k < 2; ++k)
+      if ((e = cudaEventCreateWithFlags(&h->ev_in[k], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&h->ev_att[k], cudaEventDisableTiming)) != cudaSuccess ||
+          (e = cudaEventCreateWithFlags(&h->ev_out[k], cudaEventDisableTiming)) != cudaSuccess)
+        return cuda_fail(e, "creating the step events");
   }
   const int s = h->host_slot;
   char* slot = static_cast<char*>(staging) + s * st.slot_bytes;
   char* dq = slot + 2 * (size_t)h->g.L * st.frame_bytes;
-  char* dout = static_cast<char*>(staging) + st.out_off;
+  char* dout = dq + st.q_bytes;
   const size_t fb = (size_t)nframes * h->g.N * h->g.H * h->g.D * h->g.elem;
   const size_t qb = (size_t)Lq * h->g.H * h->g.D * h->g.elem;
-  // Inputs into slot s on the copy stream, once the compute stream is done with
-  // the slot's previous contents (the call before last).
-  if (h->done_recorded[s] && (e = cudaStreamWaitEvent(h->copy_stream, h->ev_done[s], 0)) != cudaSuccess)
+  // The step follows what was enqueued on `stream` before it, unless the
+  // previous call was a step on the same stream (then `stream` only waits for
+  // that step's output, and waiting on it would serialise consecutive steps).
+  if (!(h->chained && h->chained_stream == stream)) {
+    if ((e = cudaEventRecord(h->ev_entry, stream)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(h->h2d_stream, h->ev_entry, 0)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(h->comp_stream, h->ev_entry, 0)) != cudaSuccess)
+      return cuda_fail(e, "ordering the step streams");
+  }
+  // Inputs into slot s, once the step before last has consumed them.
+  if (h->slot_used[s] && (e = cudaStreamWaitEvent(h->h2d_stream, h->ev_att[s], 0)) != cudaSuccess)
     return cuda_fail(e, "ordering the copy stream");
   for (int l = 0; l < h->g.L; ++l) {
     char* dk = slot + (size_t)(2 * l) * st.frame_bytes;
-    if ((e = cudaMemcpyAsync(dk, K_host[l], fb, cudaMemcpyHostToDevice, h->copy_stream)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dk + st.frame_bytes, V_host[l], fb, cudaMemcpyHostToDevice, h->copy_stream)) !=
+    if ((e = cudaMemcpyAsync(dk, K_host[l], fb, cudaMemcpyHostToDevice, h->h2d_stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dk + st.frame_bytes, V_host[l], fb, cudaMemcpyHostToDevice, h->h2d_stream)) !=
             cudaSuccess)
       return cuda_fail(e, "copying K/V to the device");
   }
-  if ((e = cudaMemcpyAsync(dq, Q_host, qb, cudaMemcpyHostToDevice, h->copy_stream)) != cudaSuccess)
+  if ((e = cudaMemcpyAsync(dq, Q_host, qb, cudaMemcpyHostToDevice, h->h2d_stream)) != cudaSuccess)
     return cuda_fail(e, "copying Q to the device");
-  if ((e = cudaEventRecord(h->ev_in[s], h->copy_stream)) != cudaSuccess ||
-      (e = cudaStreamWaitEvent(stream, h->ev_in[s], 0)) != cudaSuccess)
+  if ((e = cudaEventRecord(h->ev_in[s], h->h2d_stream)) != cudaSuccess ||
+      (e = cudaStreamWaitEvent(h->comp_stream, h->ev_in[s], 0)) != cudaSuccess)
     return cuda_fail(e, "ordering the compute stream");
+  // The output block of slot s is free once the step before last has copied it out.
+  if (h->slot_used[s] && (e = cudaStreamWaitEvent(h->comp_stream, h->ev_out[s], 0)) != cudaSuccess)
+    return cuda_fail(e, "ordering the compute stream");
+  void* cs = reinterpret_cast<void*>(h->comp_stream);
   fademem_status r;
   for (int l = 0; l < h->g.L; ++l) {
     char* dk = slot + (size_t)(2 * l) * st.frame_bytes;
     if ((r = fademem_insert(h, l, dk, dk + st.frame_bytes, nframes)) != FADEMEM_OK) return r;
   }
-  if ((r = fademem_consolidate(h, stream_)) != FADEMEM_OK) return r;
-  if ((r = fademem_attend(h, layer, dq, dout, Lq, stream_)) != FADEMEM_OK) return r;
-  if ((e = cudaMemcpyAsync(out_host, dout, qb, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+  if ((r = fademem_consolidate(h, cs)) != FADEMEM_OK) return r;
+  if ((r = fademem_attend(h, layer, dq, dout, Lq, cs)) != FADEMEM_OK) return r;
+  if ((e = cudaEventRecord(h->ev_att[s], h->comp_stream)) != cudaSuccess ||
+      (e = cudaStreamWaitEvent(h->d2h_stream, h->ev_att[s], 0)) != cudaSuccess)
+    return cuda_fail(e, "ordering the output copy");
+  if ((e = cudaMemcpyAsync(out_host, dout, qb, cudaMemcpyDeviceToHost, h->d2h_stream)) != cudaSuccess)
     return cuda_fail(e, "copying the output to the host");
-  if ((e = cudaEventRecord(h->ev_done[s], stream)) != cudaSuccess) return cuda_fail(e, "recording the slot event");
-  h->done_recorded[s] = true;
+  // The caller's stream continues once the output is on the host; the next
+  // step's kernels do not wait for this copy (they use the other slot).
+  if ((e = cudaEventRecord(h->ev_out[s], h->d2h_stream)) != cudaSuccess ||
+      (e = cudaStreamWaitEvent(stream, h->ev_out[s], 0)) != cudaSuccess)
+    return cuda_fail(e, "ordering the caller's stream");
+  h->slot_used[s] = true;
   h->host_slot = s ^ 1;
+  h->chained = true;
+  h->chained_stream = stream;
   return FADEMEM_OK;
 }
 
 FADEMEM_API void fademem_destroy(fademem_t h) {
   if (!h) return;
-  if (h->copy_stream) {
-    cudaStreamSynchronize(h->copy_stream);
-    cudaStreamDestroy(h->copy_stream);
+  cudaStream_t ss[3] = {h->comp_stream, h->h2d_stream, h->d2h_stream};
+  for (cudaStream_t x : ss) {
+    if (x) {
+      cudaStreamSynchronize(x);
+      cudaStreamDestroy(x);
+    }
   }
+  if (h->ev_entry) cudaEventDestroy(h->ev_entry);
   for (int s = 0; s < 2; ++s) {
     if (h->ev_in[s]) cudaEventDestroy(h->ev_in[s]);
-    if (h->ev_done[s]) cudaEventDestroy(h->ev_done[s]);
+    if (h->ev_att[s]) cudaEventDestroy(h->ev_att[s]);
+    if (h->ev_out[s]) cudaEventDestroy(h->ev_out[s]);
   }
   delete h;
 }

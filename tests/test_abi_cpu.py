@@ -119,17 +119,17 @@ def test_host_side_call_checks(cuda_lib):
 
 
 def test_host_step_staging_and_checks(cuda_lib):
-    """fademem_host_staging_bytes: two slots of (K, V per layer, Q) plus one output block, each
-    piece 256-byte aligned; fademem_step_host refuses bad arguments before any CUDA call."""
+    """fademem_host_staging_bytes: two slots of (K, V per layer, Q, output), each piece
+    256-byte aligned; fademem_step_host refuses bad arguments before any CUDA call."""
     capi.load(cuda_lib)
     lib = capi.load()
     r = lambda x: (x + 255) // 256 * 256
     cfg = _cfg(num_layers=2, tokens_per_frame=100, heads=3)
     frame = r(3 * 100 * 3 * 128 * 2)  # 3 frames of K (or V), bf16
     q = r(50 * 3 * 128 * 2)
-    assert capi.fademem_host_staging_bytes(cfg, 3, 50) == 2 * (2 * 2 * frame + q) + q
+    assert capi.fademem_host_staging_bytes(cfg, 3, 50) == 2 * (2 * 2 * frame + 2 * q)
     assert capi.fademem_host_staging_bytes(_cfg(dtype=torch.float32, num_layers=1, tokens_per_frame=7, heads=1), 1, 1) \
-        == 2 * (2 * r(7 * 128 * 4) + r(128 * 4)) + r(128 * 4)
+        == 2 * (2 * r(7 * 128 * 4) + 2 * r(128 * 4))
     for nf, lq in ((0, 50), (65, 50), (3, 0)):
         assert capi.fademem_host_staging_bytes(cfg, nf, lq) == 0
     assert capi.fademem_host_staging_bytes(_cfg(budget=1), 3, 50) == 0

@@ -273,6 +273,21 @@ def test_step_host_matches_device_path():
     for x, y in zip(a.entries(), b.entries()):
         assert np.array_equal(x, y)
     assert a.counts() == b.counts() == (M, 6 * F)
+    # Mixed with device-buffer calls on the same stream: ordering holds both ways.
+    Ks, Vs, Q = steps[0]
+    mid_a = a.attend(0, Q.cuda())
+    out_a = torch.empty((Lq, H, D), dtype=torch.bfloat16).pin_memory()
+    a.step_host(Ks, Vs, Q, out_a, layer=0)
+    tail_a = a.attend(1, Q.cuda())
+    torch.cuda.synchronize()
+    mid_b = b.attend(0, Q.cuda())
+    for l in range(L):
+        b.insert(l, Ks[l].cuda(), Vs[l].cuda())
+    b.consolidate()
+    out_b = b.attend(0, Q.cuda()).cpu()
+    tail_b = b.attend(1, Q.cuda())
+    torch.cuda.synchronize()
+    assert torch.equal(mid_a, mid_b) and torch.equal(out_a, out_b) and torch.equal(tail_a, tail_b)
     a.device_status()
     b.device_status()
 
