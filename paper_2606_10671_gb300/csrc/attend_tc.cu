@@ -468,6 +468,21 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
       // check passes, so S is still intact for the slow path.
       uint32_t pk[64];
       float rs0 = 0.f, rs1 = 0.f;
+      if (j < 2) {
+        // The group's first tile has no reference yet: take its row maximum
+        // here (a short loop), then run the same fast-path code as every other
+        // tile, which is hot in the instruction cache (the slow path is not).
+        float mx = -INFINITY;
+        for (int c = 0; c < 4; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tS + 32 * c, r);
+          tmem_ld_wait_regs(r);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
+        }
+        m_run = mx * p.scale_log2;  // finite: every tile holds at least one key
+      }
       {
         const float neg_m = -m_run;
         uint32_t r[2][32];
@@ -508,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         const float mt = mx * p.scale_log2;
         const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
         const float m_new = move ? fmaxf(mt, m_run) : m_run;
-        alpha = ex2(m_run - m_new);  // 0 on the group's first tile, 1 if unchanged
+        alpha = ex2(m_run - m_new);  // 1 if unchanged
         m_run = m_new;
         rs0 = 0.f;
         rs1 = 0.f;
