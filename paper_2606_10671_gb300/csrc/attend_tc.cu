@@ -209,22 +209,20 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-// Packed two-lane fp32 arithmetic (one instruction for two values): the
-// softmax is bound by instruction issue, so pairs halve its FFMA/FADD count.
+// Packed two-lane fp32 arithmetic (one fma.rn.f32x2 / add.rn.f32x2 for two
+// values): the softmax is bound by instruction issue, so pairs halve its
+// FFMA/FADD count.  The float2 builtins let the compiler place the pairs in
+// register pairs itself.
 __device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, float b0, float b1, float c0,
                                       float c1) {
-  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
-      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d0), "=f"(d1)
-      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+  const float2 d = __ffma2_rn(make_float2(a0, a1), make_float2(b0, b1), make_float2(c0, c1));
+  d0 = d.x;
+  d1 = d.y;
 }
 __device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d0), "=f"(d1)
-      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+  const float2 d = __fadd2_rn(make_float2(a0, a1), make_float2(b0, b1));
+  d0 = d.x;
+  d1 = d.y;
 }
 __device__ __forceinline__ float fmax3(float a, float b, float c) {
   float d;
@@ -241,13 +239,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 // most the sum, so P stays far inside bf16/fp32 range.
 constexpr float kFastRowSumLimit = 65536.f;
 
-// Exponentials of one quarter (32 keys) of this thread's row of S:
-// x = s * scale_log2 + neg_m, e = 2^x (0 for keys past `valid`), summed into
-// (rs0, rs1) and packed as bf16 pairs into pk[16 qtr .. 16 qtr + 15].
-// kRagged masks the keys past `valid` (the last tile of either key source).
+// Exponentials of one quarter (32 keys, keys 32 qtr .. 32 qtr + 31) of this
+// thread's row of S, packed into pk16 (bf16 pairs, the quarter's 16 P columns).
 template <bool kRagged>
-__device__ __forceinline__ void exp_quarter(const uint32_t (&r)[32], int qtr, int valid, float scale_log2,
-                                            float neg_m, float& rs0, float& rs1, uint32_t (&pk)[64]) {
+__device__ __forceinline__ void exp_quarter16(const uint32_t (&r)[32], int qtr, int valid, float scale_log2,
+                                              float neg_m, float& rs0, float& rs1, uint32_t (&pk16)[16]) {
 #pragma unroll
   for (int c = 0; c < 32; c += 2) {
     float x0, x1;
@@ -259,10 +255,9 @@ __device__ __forceinline__ void exp_quarter(const uint32_t (&r)[32], int qtr, in
     const float e0 = ex2(x0);
     const float e1 = ex2(x1);
     fadd2(rs0, rs1, rs0, rs1, e0, e1);
-    pk[16 * qtr + c / 2] = pack_bf16(e0, e1);
+    pk16[c / 2] = pack_bf16(e0, e1);
   }
 }
-
 __device__ __forceinline__ uint32_t barat(uint32_t bar0, int i) { return bar0 + 8u * (uint32_t)i; }
 
 __device__ __noinline__ void record_timeout(volatile int* abort_flag, unsigned int* status) {
@@ -466,51 +461,51 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
       // proves the tile safe.  The TMEM load of the next quarter of S overlaps
       // the exponentials of the current one.  P is held in registers until the
       // check passes, so S is still intact for the slow path.
-      uint32_t pk[64];
-      float rs0 = 0.f, rs1 = 0.f;
+      // The whole row of S goes to registers at once (one wait), so P can be
+      // written over S in TMEM quarter by quarter as it is computed, and the
+      // rare slow path recomputes from the registers.
+      uint32_t r[4][32];
+      tmem_ld32(tS, r[0]);
+      tmem_ld32(tS + 32, r[1]);
+      tmem_ld32(tS + 64, r[2]);
+      tmem_ld32(tS + 96, r[3]);
+      tmem_ld_wait_regs(r[0]);
+      tmem_ld_wait_regs(r[1]);
+      tmem_ld_wait_regs(r[2]);
+      tmem_ld_wait_regs(r[3]);
       if (j < 2) {
-        // The group's first tile has no reference yet: take its row maximum
-        // here (a short loop), then run the same fast-path code as every other
-        // tile, which is hot in the instruction cache (the slow path is not).
+        // The group's first tile has no reference yet: take its row maximum.
         float mx = -INFINITY;
-        for (int c = 0; c < 4; ++c) {
-          uint32_t r[32];
-          tmem_ld32(tS + 32 * c, r);
-          tmem_ld_wait_regs(r);
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
 #pragma unroll
           for (int i = 0; i < 32; ++i)
-            if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[i]));
-        }
+            if (32 * c + i < valid) mx = fmaxf(mx, __uint_as_float(r[c][i]));
         m_run = mx * p.scale_log2;  // finite: every tile holds at least one key
       }
+      // Fast path: exponentials against the running reference maximum m_run,
+      // with no max over the tile.  Any reference keeps the softmax exact (it
+      // cancels in O / l) as long as no exponential overflows, and the row sum
+      // bounds every term of the row, so a sum <= 2^16 (finite, not NaN) proves
+      // the tile safe.  P quarter q (keys 32q..32q+31) goes to P columns 16q..,
+      // which held S columns already in registers.
+      float rs0 = 0.f, rs1 = 0.f;
       {
         const float neg_m = -m_run;
-        uint32_t r[2][32];
-        tmem_ld32(tS, r[0]);
-        tmem_ld_wait_regs(r[0]);
 #pragma unroll
         for (int qtr = 0; qtr < 4; ++qtr) {
-          if (qtr < 3) tmem_ld32(tS + 32 * (qtr + 1), r[(qtr + 1) & 1]);
-          if (valid < kBN)
-            exp_quarter<true>(r[qtr & 1], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk);
-          else
-            exp_quarter<false>(r[qtr & 1], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk);
-          if (qtr < 3) tmem_ld_wait_regs(r[(qtr + 1) & 1]);
+          uint32_t pk16[16];
+          if (valid < kBN) exp_quarter16<true>(r[qtr], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk16);
+          else exp_quarter16<false>(r[qtr], qtr, valid, p.scale_log2, neg_m, rs0, rs1, pk16);
+          tmem_st16(tS + 16 * qtr, pk16);
         }
       }
       float alpha = 1.f;
       bool moved = false;
       if (__any_sync(0xffffffffu, !(rs0 + rs1 <= kFastRowSumLimit))) {
-        // Slow path (a group's first tile, or a row maximum that outgrew the
-        // reference): reload S, take the tile maximum, and move the reference
-        // lazily, only when the tile exceeds it by more than 2^8.
-        uint32_t r[4][32];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(tS + 32 * c, r[c]);
-        tmem_ld_wait_regs(r[0]);
-        tmem_ld_wait_regs(r[1]);
-        tmem_ld_wait_regs(r[2]);
-        tmem_ld_wait_regs(r[3]);
+        // Slow path (a row maximum that outgrew the reference): take the tile
+        // maximum from the registers, move the reference lazily (only when the
+        // tile exceeds it by more than 2^8) and write P again.
         float mx = -INFINITY;
 #pragma unroll
         for (int c = 0; c < 4; ++c)
@@ -521,18 +516,21 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
             mx = fmax3(mx, s0, s1);
           }
         const float mt = mx * p.scale_log2;
-        const bool move = (m_run == -INFINITY) || (mt > m_run + 8.0f);
+        const bool move = mt > m_run + 8.0f;
         const float m_new = move ? fmaxf(mt, m_run) : m_run;
         alpha = ex2(m_run - m_new);  // 1 if unchanged
         m_run = m_new;
         rs0 = 0.f;
         rs1 = 0.f;
+        tmem_st_wait();  // the fast path's stores of P land before they are overwritten
 #pragma unroll
-        for (int c = 0; c < 4; ++c) exp_quarter<true>(r[c], c, valid, p.scale_log2, -m_new, rs0, rs1, pk);
+        for (int qtr = 0; qtr < 4; ++qtr) {
+          uint32_t pk16[16];
+          exp_quarter16<true>(r[qtr], qtr, valid, p.scale_log2, -m_new, rs0, rs1, pk16);
+          tmem_st16(tS + 16 * qtr, pk16);
+        }
         moved = __any_sync(0xffffffffu, move);
       }
-      tmem_st32(tS, *reinterpret_cast<const uint32_t(*)[32]>(&pk[0]));  // P over the first 64 columns of S
-      tmem_st32(tS + 32, *reinterpret_cast<const uint32_t(*)[32]>(&pk[32]));
       l_run = l_run * alpha + (rs0 + rs1);
       if (j >= 2 && moved) {
         // Rescale O_grp before P_j V_j accumulates into it.  Its last update
