@@ -246,6 +246,16 @@ def run_cuda(args):
     t_cons = [ev[i][0].elapsed_time(ev[i][1]) for i in range(args.steps)]
     t_attn = [ev[i][1].elapsed_time(ev[i][2]) for i in range(args.steps)]
     blocks1, passes1, launches1 = mem.stats()
+    # Host cost of enqueuing one step (insert + consolidate + attend through the binding and
+    # the ABI), measured from an idle GPU on few enough steps that the launch queue never fills.
+    torch.cuda.synchronize()
+    host_us = []
+    for i in range(20):
+        h0 = time.perf_counter()
+        Q = step(i)
+        mem.attend(0, Q, out)
+        host_us.append((time.perf_counter() - h0) * 1e6)
+    torch.cuda.synchronize()
     mem.device_status()
     step_ms = max_over_ranks((sum(t_cons) + sum(t_attn)) / args.steps, dev)
     value = whole_job_rate(LQ, step_ms, ws)
@@ -305,6 +315,7 @@ def run_cuda(args):
                          "flush excluded from step time",
                    "parallelism": f"replicas x{ws} (one independent memory per GPU)"},
         "gpu_launches": launches1 - launches0,  # counted by the library
+        "host_enqueue_us_per_step": round(statistics.median(host_us), 1),  # binding + ABI calls, GPU idle
         "roofline": {"bound": "tensor", "kernel": "attend_tc_kernel", "achieved": round(attn_tflops, 1),
                      "peak": bf16_peak, "unit": "TFLOP/s", "frac": round(attn_tflops / bf16_peak, 4),
                      "peak_kind": f"{peak_kind} bf16 burst",

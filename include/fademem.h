@@ -271,6 +271,24 @@ FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void *const *K_h
                                             int nframes, int layer, const void *Q_host, void *out_host, int Lq,
                                             void *staging, size_t staging_bytes, void *stream);
 
+/* Checkpoint / resume (the paper has none; for long rollouts such as an
+ * hour-long stream).  A snapshot holds the configuration, the entry table
+ * (spans, centres, slots, frames seen) and the stored K/V of every layer;
+ * the re-indexed RoPE keys are rebuilt on import.  Snapshots are plain host
+ * bytes with a versioned header, valid across processes and devices of this
+ * library version.
+ * fademem_state_bytes: size of a snapshot of this handle (0 if h is NULL). */
+FADEMEM_API size_t fademem_state_bytes(fademem_t h);
+/* Write a snapshot into host memory (>= fademem_state_bytes).  Synchronises
+ * stream first.  Errors: INVALID_ARG, PENDING (frames inserted but not
+ * consolidated), WORKSPACE (buffer too small), CUDA. */
+FADEMEM_API fademem_status fademem_export_state(fademem_t h, void *host_buf, size_t bytes, void *stream);
+/* Replace this handle's memory with a snapshot taken from a handle of the
+ * same configuration (every fademem_config field equal).  Any pending frames
+ * are dropped.  Synchronises stream.  Errors: INVALID_ARG (not a snapshot,
+ * other version, other configuration, inconsistent contents), CUDA. */
+FADEMEM_API fademem_status fademem_import_state(fademem_t h, const void *host_buf, size_t bytes, void *stream);
+
 /* Release the handle (NULL-safe).  Does not free the caller's workspace. */
 FADEMEM_API void fademem_destroy(fademem_t h);
 

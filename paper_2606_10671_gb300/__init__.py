@@ -175,6 +175,14 @@ class FadeMem:
     def device_status(self, stream=None, raise_on_error=True):
         return capi.fademem_get_device_status(self.handle, _stream_handle(stream), raise_on_error)
 
+    def export_state(self, stream=None):
+        """Snapshot of the memory (entry table and stored K/V of every layer) as host bytes."""
+        return capi.fademem_export_state(self.handle, _stream_handle(stream))
+
+    def import_state(self, snapshot, stream=None):
+        """Replace the memory with a snapshot from a memory of the same configuration."""
+        capi.fademem_import_state(self.handle, snapshot, _stream_handle(stream))
+
     def reset(self, stream=None):
         capi.fademem_reset(self.handle, _stream_handle(stream))
 

@@ -36,7 +36,8 @@ EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fadem
            "fademem_counts", "fademem_get_entries", "fademem_last_plan", "fademem_stats",
            "fademem_layer_memory", "fademem_get_device_status",
            "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc",
-           "fademem_host_staging_bytes", "fademem_step_host", "fademem_destroy", "fademem_last_error")
+           "fademem_host_staging_bytes", "fademem_step_host", "fademem_state_bytes", "fademem_export_state",
+           "fademem_import_state", "fademem_destroy", "fademem_last_error")
 
 
 class fademem_config(ctypes.Structure):
@@ -88,6 +89,9 @@ def load(path: str | None = None):
             "fademem_consolidate_noalloc": (I, [P, P]),
             "fademem_host_staging_bytes": (ctypes.c_size_t, [cfgp, I, I]),
             "fademem_step_host": (I, [P, ctypes.POINTER(P), ctypes.POINTER(P), I, I, P, P, I, P, ctypes.c_size_t, P]),
+            "fademem_state_bytes": (ctypes.c_size_t, [P]),
+            "fademem_export_state": (I, [P, P, ctypes.c_size_t, P]),
+            "fademem_import_state": (I, [P, P, ctypes.c_size_t, P]),
             "fademem_destroy": (None, [P]),
             "fademem_last_error": (ctypes.c_char_p, []),
         }
@@ -208,6 +212,24 @@ def fademem_step_host(h: int, K_host, V_host, nframes: int, layer: int, Q_host: 
     check(load().fademem_step_host(ctypes.c_void_p(h), Ks, Vs, nframes, layer, ctypes.c_void_p(Q_host),
                                    ctypes.c_void_p(out_host), Lq, ctypes.c_void_p(staging), staging_bytes,
                                    ctypes.c_void_p(stream)))
+
+
+def fademem_state_bytes(h: int) -> int:
+    return int(load().fademem_state_bytes(ctypes.c_void_p(h)))
+
+
+def fademem_export_state(h: int, stream: int = 0):
+    """A snapshot of the memory as a numpy uint8 array."""
+    import numpy as np
+    buf = np.empty(fademem_state_bytes(h), np.uint8)
+    check(load().fademem_export_state(ctypes.c_void_p(h), buf.ctypes.data, buf.size, ctypes.c_void_p(stream)))
+    return buf
+
+
+def fademem_import_state(h: int, snapshot, stream: int = 0):
+    import numpy as np
+    buf = np.ascontiguousarray(np.frombuffer(snapshot, np.uint8))
+    check(load().fademem_import_state(ctypes.c_void_p(h), buf.ctypes.data, buf.size, ctypes.c_void_p(stream)))
 
 
 def fademem_destroy(h: int):

@@ -10,6 +10,8 @@
 #include <new>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "fademem_internal.h"
 
 using namespace fademem;
@@ -17,6 +19,15 @@ using namespace fademem;
 namespace {
 
 thread_local char g_err[512] = "";
+
+// NVTX range around an entry point, visible in Nsight timelines (a no-op
+// unless a tool is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 fademem_status fail(fademem_status s, const char* fmt, ...) {
   va_list ap;
@@ -153,6 +164,7 @@ FADEMEM_API fademem_status fademem_create(const fademem_config* cfg, void* works
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "out of host memory");
   h->cfg = *cfg;
   if (h->cfg.scale == 0.f) h->cfg.scale = 1.0f / sqrtf((float)cfg->head_dim);
+  if (h->cfg.rope_pairs > 0 && h->cfg.rope_theta == 0.0) h->cfg.rope_theta = 10000.0;  // the documented default
   h->g = g;
   h->ws = reinterpret_cast<char*>(workspace);
   h->ws_bytes = workspace_bytes;
@@ -174,6 +186,7 @@ FADEMEM_API fademem_status fademem_create(const fademem_config* cfg, void* works
 }
 
 FADEMEM_API fademem_status fademem_insert(fademem_t h, int layer, const void* K, const void* V, int nframes) {
+  NvtxRange nvtx_("fademem_insert");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
   if (!K || !V) return fail(FADEMEM_ERR_INVALID_ARG, "K or V is NULL");
@@ -201,6 +214,7 @@ static fademem_status ensure_init(fademem_t h, cudaStream_t stream) {
 
 
 FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
+  NvtxRange nvtx_("fademem_consolidate");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->chained = false;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
@@ -309,6 +323,7 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
 
 static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const void* Kcur, const void* Vcur,
                                   int ncur, void* out, int Lq, void* stream_) {
+  NvtxRange nvtx_(ncur > 0 ? "fademem_attend_ext" : "fademem_attend");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->chained = false;
   if (layer < 0 || layer >= h->g.L) return fail(FADEMEM_ERR_INVALID_ARG, "layer %d out of range", layer);
@@ -461,6 +476,7 @@ FADEMEM_API fademem_status fademem_selftest_wait_timeout(fademem_t h, void* stre
 }
 
 FADEMEM_API fademem_status fademem_reset(fademem_t h, void* stream_) {
+  NvtxRange nvtx_("fademem_reset");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->chained = false;
   h->la_valid = false;
@@ -513,6 +529,7 @@ fademem_status noalloc_scratch(DevState** out) {
 extern "C" {
 
 FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream_) {
+  NvtxRange nvtx_("fademem_consolidate_noalloc");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->chained = false;
   if (h->g.M + 1 > kMaxEntries)
@@ -566,6 +583,7 @@ FADEMEM_API size_t fademem_host_staging_bytes(const fademem_config* cfg, int nfr
 FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void* const* K_host, const void* const* V_host,
                                             int nframes, int layer, const void* Q_host, void* out_host, int Lq,
                                             void* staging, size_t staging_bytes, void* stream_) {
+  NvtxRange nvtx_("fademem_step_host");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   if (!K_host || !V_host || !Q_host || !out_host) return fail(FADEMEM_ERR_INVALID_ARG, "a host pointer is NULL");
   for (int l = 0; l < h->g.L; ++l)
@@ -647,6 +665,126 @@ FADEMEM_API fademem_status fademem_step_host(fademem_t h, const void* const* K_h
   h->host_slot = s ^ 1;
   h->chained = true;
   h->chained_stream = stream;
+  return FADEMEM_OK;
+}
+
+// Snapshot layout: SnapshotHeader, then the entry table (DevMeta), then for
+// every layer its stored K and V blocks ([H][M][N][D] each), all packed.
+struct SnapshotHeader {
+  char magic[8];            // "FADEMEM" + '\0'
+  uint32_t version;         // 1
+  uint32_t header_bytes;    // sizeof(SnapshotHeader)
+  fademem_config cfg;
+  int32_t count;
+  int32_t pad;
+  int64_t frames;
+  uint64_t meta_bytes;      // sizeof(DevMeta)
+  uint64_t kv_bytes;        // bytes of one layer's K (or V) block
+};
+static const char kSnapshotMagic[8] = {'F', 'A', 'D', 'E', 'M', 'E', 'M', 0};
+
+static bool same_config(const fademem_config& a, const fademem_config& b) {
+  return a.budget == b.budget && a.heads == b.heads && a.head_dim == b.head_dim &&
+         a.tokens_per_frame == b.tokens_per_frame && a.num_layers == b.num_layers && a.beta == b.beta &&
+         a.anchor == b.anchor && a.merge_op == b.merge_op && a.dtype == b.dtype && a.scale == b.scale &&
+         a.rope_pairs == b.rope_pairs && (a.rope_pairs == 0 || a.rope_theta == b.rope_theta);
+}
+
+FADEMEM_API size_t fademem_state_bytes(fademem_t h) {
+  if (!h) return 0;
+  return sizeof(SnapshotHeader) + sizeof(DevMeta) + 2 * (size_t)h->g.L * h->g.kv_elems * h->g.elem;
+}
+
+FADEMEM_API fademem_status fademem_export_state(fademem_t h, void* host_buf, size_t bytes, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (!host_buf) return fail(FADEMEM_ERR_INVALID_ARG, "host buffer is NULL");
+  if (bytes < fademem_state_bytes(h))
+    return fail(FADEMEM_ERR_WORKSPACE, "snapshot needs %zu bytes (got %zu)", fademem_state_bytes(h), bytes);
+  for (int l = 0; l < h->g.L; ++l)
+    if (h->pending_frames[l] != 0)
+      return fail(FADEMEM_ERR_PENDING, "frames inserted on layer %d await fademem_consolidate", l);
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  fademem_status s = ensure_init(h, stream);
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  char* out = static_cast<char*>(host_buf);
+  SnapshotHeader hd;
+  memset(&hd, 0, sizeof(hd));
+  memcpy(hd.magic, kSnapshotMagic, sizeof(hd.magic));
+  hd.version = 1;
+  hd.header_bytes = sizeof(SnapshotHeader);
+  hd.cfg = h->cfg;
+  hd.count = h->count;
+  hd.frames = h->frames;
+  hd.meta_bytes = sizeof(DevMeta);
+  hd.kv_bytes = h->g.kv_elems * h->g.elem;
+  memcpy(out, &hd, sizeof(hd));
+  out += sizeof(hd);
+  if ((e = cudaMemcpy(out, &cur_state(h)->meta, sizeof(DevMeta), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "reading the entry table");
+  out += sizeof(DevMeta);
+  for (int l = 0; l < h->g.L; ++l) {
+    const char* Kl = h->cache + (size_t)l * h->g.layer_bytes;
+    if ((e = cudaMemcpy(out, Kl, 2 * hd.kv_bytes, cudaMemcpyDeviceToHost)) != cudaSuccess)
+      return cuda_fail(e, "reading the memory");
+    out += 2 * hd.kv_bytes;
+  }
+  return FADEMEM_OK;
+}
+
+FADEMEM_API fademem_status fademem_import_state(fademem_t h, const void* host_buf, size_t bytes, void* stream_) {
+  if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
+  if (!host_buf) return fail(FADEMEM_ERR_INVALID_ARG, "host buffer is NULL");
+  if (bytes < sizeof(SnapshotHeader)) return fail(FADEMEM_ERR_INVALID_ARG, "not a FadeMem snapshot (too short)");
+  SnapshotHeader hd;
+  memcpy(&hd, host_buf, sizeof(hd));
+  if (memcmp(hd.magic, kSnapshotMagic, sizeof(hd.magic)) != 0)
+    return fail(FADEMEM_ERR_INVALID_ARG, "not a FadeMem snapshot (bad magic)");
+  if (hd.version != 1 || hd.header_bytes != sizeof(SnapshotHeader) || hd.meta_bytes != sizeof(DevMeta))
+    return fail(FADEMEM_ERR_INVALID_ARG, "snapshot of another library version (%u)", hd.version);
+  if (!same_config(hd.cfg, h->cfg)) return fail(FADEMEM_ERR_INVALID_ARG, "snapshot of another configuration");
+  if (hd.kv_bytes != h->g.kv_elems * h->g.elem || bytes < fademem_state_bytes(h))
+    return fail(FADEMEM_ERR_INVALID_ARG, "snapshot size does not match the configuration");
+  const char* in = static_cast<const char*>(host_buf) + sizeof(hd);
+  DevMeta meta;
+  memcpy(&meta, in, sizeof(meta));
+  in += sizeof(meta);
+  const long long expect = hd.frames < h->g.M ? hd.frames : h->g.M;
+  if (hd.frames < 0 || hd.count != expect || meta.count != hd.count || meta.t_next != hd.frames)
+    return fail(FADEMEM_ERR_INVALID_ARG, "snapshot entry table is inconsistent (count %d, frames %lld)", hd.count,
+                (long long)hd.frames);
+  for (int i = 0; i < meta.count; ++i)
+    if (meta.slot[i] < 0 || meta.slot[i] >= h->g.M)
+      return fail(FADEMEM_ERR_INVALID_ARG, "snapshot entry %d has slot %d", i, meta.slot[i]);
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  h->chained = false;
+  h->need_init = true;
+  fademem_status s = ensure_init(h, stream);  // clears the status word, counters and both entry tables
+  if (s != FADEMEM_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "synchronising the stream");
+  if ((e = cudaMemcpy(&cur_state(h)->meta, &meta, sizeof(meta), cudaMemcpyHostToDevice)) != cudaSuccess)
+    return cuda_fail(e, "writing the entry table");
+  for (int l = 0; l < h->g.L; ++l) {
+    char* Kl = h->cache + (size_t)l * h->g.layer_bytes;
+    if ((e = cudaMemcpy(Kl, in, 2 * hd.kv_bytes, cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "writing the memory");
+    in += 2 * hd.kv_bytes;
+  }
+  for (int l = 0; l < h->g.L; ++l) {
+    h->pending[l].clear();
+    h->pending_frames[l] = 0;
+  }
+  h->count = hd.count;
+  h->frames = hd.frames;
+  h->la_valid = false;
+  if (h->g.rope_pairs > 0 && h->count > 0) {
+    e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "launching the re-phase kernel");
+    ++h->launches;
+    if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "rebuilding the attention keys");
+  }
   return FADEMEM_OK;
 }
 

@@ -22,7 +22,7 @@ def _declared_symbols():
 def test_exports_every_declared_symbol(cuda_lib):
     lib = ctypes.CDLL(cuda_lib)
     declared = _declared_symbols()
-    assert len(declared) == 19
+    assert len(declared) == 22
     for name in declared:
         assert hasattr(lib, name), name
     assert sorted(capi.EXPORTS) == declared
@@ -167,4 +167,34 @@ def test_cuda_failure_is_a_status(cuda_lib):
     assert lib.fademem_insert(P(h), 0, P(FAKE_WS), P(FAKE_WS), 3) == capi.FADEMEM_OK
     assert lib.fademem_consolidate(P(h), None) == capi.FADEMEM_ERR_CUDA
     assert "cuda" in capi.fademem_last_error().lower()
+    capi.fademem_destroy(h)
+
+
+def test_snapshot_size_and_import_checks(cuda_lib):
+    """fademem_state_bytes = header + entry table + K and V of every layer; imports of
+    anything but a snapshot of the same configuration are refused before any CUDA call."""
+    import struct
+    capi.load(cuda_lib)
+    lib = capi.load()
+    cfg = _cfg(num_layers=2, tokens_per_frame=64, heads=2)
+    st, h = _create_status(cfg)
+    assert st == capi.FADEMEM_OK
+    kv = 2 * 21 * 64 * 128 * 2  # one layer's K block: H*M*N*D bf16
+    n = capi.fademem_state_bytes(h)
+    overhead = n - 2 * 2 * kv
+    assert 0 < overhead < 8192
+    assert capi.fademem_state_bytes(None) == 0
+    P = ctypes.c_void_p
+    junk = (ctypes.c_char * n)()
+    assert lib.fademem_import_state(P(h), junk, n, None) == capi.FADEMEM_ERR_INVALID_ARG
+    assert "magic" in capi.fademem_last_error()
+    assert lib.fademem_import_state(P(h), junk, 16, None) == capi.FADEMEM_ERR_INVALID_ARG
+    # a header with the right magic and version but another configuration
+    other = _cfg(num_layers=2, tokens_per_frame=64, heads=2, beta=0.5)
+    hdr = b"FADEMEM\0" + struct.pack("<II", 1, 0) + bytes(other)
+    buf = (ctypes.c_char * n).from_buffer_copy(hdr + b"\0" * (n - len(hdr)))
+    st = lib.fademem_import_state(P(h), buf, n, None)
+    assert st == capi.FADEMEM_ERR_INVALID_ARG
+    assert lib.fademem_export_state(P(h), None, n, None) == capi.FADEMEM_ERR_INVALID_ARG
+    assert lib.fademem_export_state(P(h), junk, n - 1, None) == capi.FADEMEM_ERR_WORKSPACE
     capi.fademem_destroy(h)

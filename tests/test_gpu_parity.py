@@ -383,3 +383,35 @@ def test_attention_reference_moves(qscale):
     ref = ref_mem.attend_ext(Q.double().cpu().numpy(), Kc.double().cpu().numpy(), Vc.double().cpu().numpy(), N, H, D)
     assert_close(out.double().cpu().numpy(), ref, torch.bfloat16, "sharp attention + chunk")
     p.gpu.device_status()
+
+
+@pytest.mark.parametrize("dtype,rope", [(torch.float32, 0), (torch.bfloat16, 22)])
+def test_export_import_resume(dtype, rope):
+    """Checkpoint / resume: a memory restored from a snapshot into a fresh handle and the
+    original, fed the same frames afterwards, stay bit-identical (entries, stored K/V,
+    attention with RoPE keys rebuilt), and both still match the oracle."""
+    from paper_2606_10671_gb300 import FadeMem
+    D, N, M = 128, 40, 6
+    p = Pair(M, 2, D, N, beta=0.3, dtype=dtype, seed=31, rope_pairs=rope)
+    for seg in range(5):
+        p.step(3)
+    snap = p.gpu.export_state()
+    q = FadeMem(M, 2, D, N, beta=0.3, dtype=dtype, rope_pairs=rope)
+    q.import_state(snap)
+    assert q.counts() == p.gpu.counts()
+    for seg in range(4):
+        p.insert(3)
+        for l in range(p.L):
+            K, V = p._keep[l]
+            q.insert(l, K, V)
+        p.gpu.consolidate()
+        q.consolidate()
+        for x, y in zip(p.gpu.entries(), q.entries()):
+            assert np.array_equal(x, y)
+        for a, b in zip(p.gpu.layer_memory(0), q.layer_memory(0)):
+            assert torch.equal(a, b)
+    Q = p.queries(70, step=2)
+    assert torch.equal(p.gpu.attend(0, Q), q.attend(0, Q))
+    p.check_entries()
+    p.check_attend(Q)
+    q.device_status()
