@@ -38,7 +38,9 @@ def _load():
     with _lock:
         if _lib is not None:
             return _lib
-        lib = ctypes.CDLL(build_oracle())
+        # FADEMEM_ORACLE_LIB: a separately built oracle (the sanitizer tests build one
+        # with ASan/UBSan and run the pins against it).
+        lib = ctypes.CDLL(os.environ.get("FADEMEM_ORACLE_LIB") or build_oracle())
         P = ctypes.c_void_p
         dp = ctypes.POINTER(ctypes.c_double)
         lib.oracle_create.restype = P

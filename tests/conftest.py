@@ -21,6 +21,7 @@ def oracle_lib():
 
 @pytest.fixture(scope="session")
 def cuda_lib():
-    """The CUDA library, built in-tree if missing (nvcc cross-compiles without a GPU)."""
+    """The CUDA library, built in-tree if missing (nvcc cross-compiles without a GPU).
+    FADEMEM_CUDA_LIB names another build (the sanitizer tests use one built with ASan/UBSan)."""
     from paper_2606_10671_gb300 import build
-    return build.build_library()
+    return os.environ.get("FADEMEM_CUDA_LIB") or build.build_library()
