@@ -58,6 +58,24 @@ def test_bf16_attention_edges(N, Lq, frames):
     p.check_attend(p.queries(Lq, step=1))
 
 
+@pytest.mark.parametrize("M,N,H,Lq,ncur", [(5, 1000, 3, 300, 0), (4, 1100, 3, 200, 0), (5, 700, 2, 300, 2100),
+                                            (5, 1000, 8, 2560, 0)])
+def test_bf16_long_key_rows_few_query_tiles(M, N, H, Lq, ncur):
+    """Few query tiles (6-9, far below one CTA per SM) over 35-45 key tiles each,
+    ragged in both the memory and the chunk keys; and (H=8, Lq=2560) 160 query
+    tiles, a little over one wave, with sampled rows on tile edges."""
+    p = Pair(M, H, 128, N, beta=0.3, dtype=torch.bfloat16, seed=21, tracked_heads=list(range(min(H, 3))))
+    rows = None if Lq <= 300 else np.array([0, 127, 128, 1000, 2047, 2048, 2559])
+    for seg in range(3):
+        p.step(3)
+        if ncur:
+            Kc, Vc = p.chunk(ncur, step=seg)
+            p.check_attend_ext(p.queries(Lq, step=seg), Kc, Vc, rows=rows)
+        else:
+            p.check_attend(p.queries(Lq, step=seg), rows=rows)
+    p.gpu.device_status()
+
+
 @pytest.mark.parametrize("op", ["weighted", "average", "select_nearest", "max_pool"])
 @pytest.mark.parametrize("anchor", [True, False])
 def test_merge_operators_fp32(op, anchor):
