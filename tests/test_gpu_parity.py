@@ -403,6 +403,91 @@ def test_attention_reference_moves(qscale):
     p.gpu.device_status()
 
 
+@pytest.mark.parametrize("huge", [(5, 7), (4, 6), (4, 5, 7)])
+def test_attention_reference_moves_inside_a_tile(huge):
+    """One 64-token frame per half key tile (slot 2j: keys 0-63 of tile j, slot 2j+1:
+    keys 64-127), no merges.  The frames in `huge` have keys scaled by 40, so their
+    scores sit ~2^130 above the reference that each softmax group takes from its first
+    tile (tiles 0 and 1 stay ordinary): exponentials against the old reference overflow
+    and the kernel must move its reference.  (5, 7): only keys 64-127 of the groups'
+    second tiles jump; (4, 6): only keys 0-63; (4, 5, 7): both halves, and a lone
+    second half.  Compared with the oracle's attention over the same bf16 keys."""
+    from oracle import OracleMemory
+    from paper_2606_10671_gb300 import FadeMem
+    N, H, D, F = 64, 2, 128, 8
+    g = np.random.default_rng([31, len(huge)] + list(huge))
+    K = g.standard_normal((F, N, H, D), dtype=np.float32)
+    V = g.standard_normal((F, N, H, D), dtype=np.float32)
+    for f in huge:
+        K[f] *= 40.0
+    Kb = torch.from_numpy(K).to(torch.bfloat16)
+    Vb = torch.from_numpy(V).to(torch.bfloat16)
+    mem = FadeMem(F, H, D, N, num_layers=1, beta=0.3, dtype=torch.bfloat16)
+    mem.insert(0, Kb.reshape(F * N, H, D).cuda(), Vb.reshape(F * N, H, D).cuda())
+    mem.consolidate()
+    slot = mem.entries()[0]
+    assert slot.tolist() == list(range(F))  # frame f in slot f: key tile j = frames 2j, 2j+1
+    ref_mem = OracleMemory(F + 1, 0.3, elems=N * H * D)
+    for f in range(F):
+        ref_mem.insert(Kb[f].double().numpy(), Vb[f].double().numpy())
+    Q = torch.from_numpy(g.standard_normal((200, H, D), dtype=np.float32)).to(torch.bfloat16)
+    out = mem.attend(0, Q.cuda())
+    torch.cuda.synchronize()
+    ref = ref_mem.attend(Q.double().numpy(), N, H, D)
+    assert_close(out.double().cpu().numpy(), ref, torch.bfloat16, "reference moved inside a tile")
+    mem.device_status()
+
+
+@pytest.mark.parametrize("dtype,D", [(torch.bfloat16, 128), (torch.float32, 64)])
+def test_attend_captured_in_cuda_graph(dtype, D):
+    """A segment's denoising-step attends (2 layers x 4 steps, one with a current
+    chunk) captured once in a CUDA graph, then replayed twice with new queries written
+    into the captured input buffers: outputs bit-identical to eager calls on the same
+    queries (the attention kernels are deterministic and keep no host state)."""
+    from paper_2606_10671_gb300 import FadeMem
+    H, N, Lq, L = 4, 200, 300, 2
+    gen = torch.Generator(device="cuda").manual_seed(5)
+    rnd = lambda *shape: torch.randn(*shape, device="cuda", generator=gen).to(dtype)
+    mem = FadeMem(5, H, D, N, num_layers=L, beta=0.3, dtype=dtype)
+    for seg in range(4):
+        for layer in range(L):
+            mem.insert(layer, rnd(3 * N, H, D), rnd(3 * N, H, D))
+        mem.consolidate()
+    Kc, Vc = rnd(3 * N, H, D), rnd(3 * N, H, D)
+    Qs = [[rnd(Lq, H, D) for _ in range(4)] for _ in range(L)]
+    outs = [[torch.empty_like(Qs[0][0]) for _ in range(4)] for _ in range(L)]
+
+    def steps():
+        for layer in range(L):
+            for k in range(4):
+                if k == 3:
+                    mem.attend_ext(layer, Qs[layer][k], Kc, Vc, out=outs[layer][k])
+                else:
+                    mem.attend(layer, Qs[layer][k], out=outs[layer][k])
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        steps()  # warm-up outside the capture (first-call set-up)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        steps()
+    for rep in range(2):
+        for layer in range(L):
+            for k in range(4):
+                Qs[layer][k].copy_(rnd(Lq, H, D))
+        graph.replay()
+        torch.cuda.synchronize()
+        for layer in range(L):
+            for k in range(4):
+                ref = (mem.attend_ext(layer, Qs[layer][k], Kc, Vc) if k == 3 else mem.attend(layer, Qs[layer][k]))
+                torch.cuda.synchronize()
+                assert torch.equal(outs[layer][k], ref), (rep, layer, k)
+    mem.device_status()
+
+
 @pytest.mark.parametrize("dtype,rope", [(torch.float32, 0), (torch.bfloat16, 22)])
 def test_export_import_resume(dtype, rope):
     """Checkpoint / resume: a memory restored from a snapshot into a fresh handle and the
