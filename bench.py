@@ -273,7 +273,9 @@ def run_cuda(args):
     Lk = M * N
     flops = 4.0 * LQ * Lk * H * D
     attn_tflops = flops / (attn_ms / 1e3) / 1e12
-    cons_bytes = (blocks1 - blocks0) * block_bytes / max(1, passes1 - passes0)  # mean per pass (= per step)
+    # Mean per step (one fademem_consolidate call of 3 frames = one pass).  It falls slowly over a
+    # long run: anchor merges, which move no bytes, grow more frequent as the history lengthens.
+    cons_bytes = (blocks1 - blocks0) * block_bytes / args.steps
     cons_gbs = cons_bytes / (cons_ms / 1e3) / 1e9
 
     # End to end through the C ABI with host buffers: fademem_step_host copies each step's
@@ -333,7 +335,8 @@ def run_cuda(args):
                         "frac": round(cons_gbs / hbm_peak, 4), "bytes_per_step": round(cons_bytes),
                         "frac_of_nominal": round(cons_gbs / NOMINAL_HBM_GBS, 4), "nominal_gbs": NOMINAL_HBM_GBS,
                         "ms_per_step": round(cons_ms, 4),
-                        "blocks_per_step": round((blocks1 - blocks0) / max(1, passes1 - passes0), 3),
+                        "blocks_per_step": round((blocks1 - blocks0) / args.steps, 3),
+                        "passes_per_step": round((passes1 - passes0) / args.steps, 3),
                         "note": "event time of the fademem_consolidate call (in steady state the consolidation "
                                 "kernel alone: the next pass is scheduled inside it); algorithmic bytes from the "
                                 "device's own count of blocks moved over the timed steps",
