@@ -438,6 +438,43 @@ def test_attention_reference_moves_inside_a_tile(huge):
     mem.device_status()
 
 
+def _fuzz_case(i):
+    """Case i of the seeded fuzz: a small random configuration and call pattern."""
+    rng = np.random.default_rng([4242, i])
+    dtype = torch.bfloat16 if rng.integers(0, 2) else torch.float32
+    D = 128 if dtype == torch.bfloat16 else int(rng.choice([64, 128]))
+    return dict(dtype=dtype, D=D, M=int(rng.integers(2, 12)), H=int(rng.integers(1, 4)),
+                N=int(rng.integers(1, 300)), beta=float(rng.choice([0.1, 0.3, 0.5, 0.7, 0.9, 1.0])),
+                anchor=bool(rng.integers(0, 2)),
+                op=str(rng.choice(["weighted", "average", "select_nearest", "max_pool"])),
+                rope=int(rng.choice([0, 0, 8, D // 2])), frames=int(rng.integers(1, 8)),
+                per_call=int(rng.integers(1, 5)), segments=int(rng.integers(3, 9)), Lq=int(rng.integers(1, 400)),
+                ncur=int(rng.integers(0, 500)), seed=int(rng.integers(0, 1 << 30)))
+
+
+@pytest.mark.parametrize("case", range(48))
+def test_fuzz_small_configurations(case):
+    """Seeded random small configurations covering every option together:
+    - budget 2-11, 1-3 heads, 1-299 tokens per frame;
+    - beta from {0.1, 0.3, 0.5, 0.7, 0.9, 1}, anchor on or off, all four merge operators;
+    - fp32 (D 64 or 128) or bf16, temporal RoPE off or on;
+    - 1-7 frames per segment inserted in calls of 1-4 frames.
+    After every segment the entry table must be bit-exact and every stored
+    block within tolerance; then attention over the memory, and over the
+    memory plus a random current chunk, against the oracle."""
+    c = _fuzz_case(case)
+    p = Pair(c["M"], c["H"], c["D"], c["N"], beta=c["beta"], anchor=c["anchor"], op=c["op"], dtype=c["dtype"],
+             seed=c["seed"], rope_pairs=c["rope"])
+    for seg in range(c["segments"]):
+        p.step(c["frames"], per_call=c["per_call"])
+        p.check_entries()
+        p.check_memory()
+    p.check_attend(p.queries(c["Lq"], step=seg))
+    Kc, Vc = p.chunk(c["ncur"], step=seg)
+    p.check_attend_ext(p.queries(c["Lq"], step=seg + 1), Kc, Vc)
+    p.gpu.device_status()
+
+
 @pytest.mark.parametrize("dtype,D", [(torch.bfloat16, 128), (torch.float32, 64)])
 def test_attend_captured_in_cuda_graph(dtype, D):
     """A segment's denoising-step attends (2 layers x 4 steps, one with a current
