@@ -48,6 +48,12 @@ extern "C" {
 /* Largest number of frames pending (inserted, not yet consolidated) per layer. */
 #define FADEMEM_MAX_PENDING 64
 
+/* Bits of the device status word (fademem_get_device_status). */
+#define FADEMEM_STATUS_TIMEOUT 0x1u
+#define FADEMEM_STATUS_COUNT_MISMATCH 0x2u
+#define FADEMEM_STATUS_PLAN_OVERFLOW 0x4u
+#define FADEMEM_STATUS_NEAR_TIE 0x8u
+
 typedef enum fademem_status {
     FADEMEM_OK = 0,
     FADEMEM_ERR_INVALID_ARG = 1,    /* NULL / misaligned pointer, out-of-range size or index */
@@ -197,7 +203,20 @@ FADEMEM_API fademem_status fademem_layer_memory(fademem_t h, int layer, void **K
 
 /* Read and clear the device status word (synchronises stream).  Returns OK,
  * DEVICE_TIMEOUT (a bounded wait in a kernel gave up) or DEVICE_CHECK; the
- * raw word goes to *word when word is not NULL. */
+ * raw word goes to *word when word is not NULL.  Bits of the word:
+ *   FADEMEM_STATUS_TIMEOUT         a bounded device wait gave up;
+ *   FADEMEM_STATUS_COUNT_MISMATCH  host and device entry counts disagreed;
+ *   FADEMEM_STATUS_PLAN_OVERFLOW   a merge plan exceeded its static bounds;
+ *   FADEMEM_STATUS_NEAR_TIE        a schedule decision of Algorithm S1 (the
+ *     argmin of the warped gaps, Sec. 3.3) was not certified: its best and
+ *     second-best gaps were equal within the fp64 evaluation error of d^beta
+ *     (2^-48 of the sum of the four u values involved) and not exactly
+ *     computable (beta = 1, or beta = 0.5 on exact square roots, are).  The
+ *     decision taken (lowest index among the equal minima) is a valid one,
+ *     but another fp64 evaluation of d^beta, such as a host libm's, may
+ *     choose the other pair.  The message names the first such frame.
+ * Every other configuration decides each merge exactly as an fp64 evaluation
+ * of Algorithm S1 does. */
 FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void *stream, uint32_t *word);
 
 /* Diagnostic of device-side failure detection: enqueues one thread that waits,
@@ -231,9 +250,10 @@ FADEMEM_API fademem_status fademem_reset(fademem_t h, void *stream);
  * stream capture.  Every call shares the one array: calls that overlap on the
  * GPU (other streams, other handles, other threads) race and must be
  * serialised by the caller.  Nothing in the array needs clearing: each call
- * overwrites it from the handle's workspace before use.  A handle whose entry
- * table would not fit the array (budget above FADEMEM_MAX_BUDGET) is rejected
- * with FADEMEM_ERR_UNSUPPORTED.  Other errors as fademem_consolidate. */
+ * overwrites it from the handle's workspace before use.  The array holds the
+ * entry table of every budget fademem_create accepts (up to
+ * FADEMEM_MAX_BUDGET; checked when the library is compiled).  Errors as
+ * fademem_consolidate. */
 FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void *stream);
 
 /* Device staging bytes fademem_step_host needs for segments of `nframes`

@@ -27,7 +27,7 @@
  *      per head: out = softmax(scale * q K^T) V (the backbone attention whose
  *      context the memory supplies, Sec. 3.3 last paragraph, Sec. 4.1).
  *
- * Readings where the paper is silent (each one also listed in the design notes):
+ * Readings where the paper is silent:
  *   - frames are numbered from t = 0, so the anchor's own centre is mu = 0;
  *   - ties in the argmin go to the lowest pair index (the oldest pair);
  *   - the anchor is entry 0; its pair is j == 0;

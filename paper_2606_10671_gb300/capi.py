@@ -21,6 +21,11 @@ FADEMEM_ERR_PENDING = 5
 FADEMEM_ERR_CUDA = 6
 FADEMEM_ERR_DEVICE_TIMEOUT = 7
 FADEMEM_ERR_DEVICE_CHECK = 8
+# Bits of the device status word (include/fademem.h, FADEMEM_STATUS_*).
+STATUS_TIMEOUT = 0x1
+STATUS_COUNT_MISMATCH = 0x2
+STATUS_PLAN_OVERFLOW = 0x4
+STATUS_NEAR_TIE = 0x8
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "WORKSPACE", 4: "EMPTY", 5: "PENDING", 6: "CUDA",
                 7: "DEVICE_TIMEOUT", 8: "DEVICE_CHECK"}
 

@@ -27,6 +27,7 @@
 #include <stdio.h>
 
 #include "fademem_internal.h"
+#include "per_device.h"
 
 namespace fademem {
 namespace {
@@ -670,11 +671,19 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
     snprintf(err, errlen, "cuTensorMapEncodeTiled is unavailable from the driver");
     return cudaErrorNotSupported;
   }
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(attend_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  {
+    // The shared-memory opt-in is a per-device setting: once per device, with it current.
+    static PerDevice<char> smem_opt_in;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    char done = 0;
+    if (!smem_opt_in.get(dev, [&e](int, char* v) {
+          e = cudaFuncSetAttribute(attend_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+          *v = 1;
+          return e == cudaSuccess;
+        }, &done))
+      return e != cudaSuccess ? e : cudaErrorInvalidDevice;
   }
   AttnParams prm;
   const uint64_t row = (uint64_t)kHD * 2;

@@ -19,6 +19,7 @@
 #include <math.h>
 
 #include "fademem_internal.h"
+#include "per_device.h"
 
 namespace fademem {
 namespace {
@@ -40,6 +41,9 @@ __device__ __forceinline__ float warp_u32(float d, float beta) {
   return powf(d, beta);
 }
 constexpr float kU32RelErr = 1.0f / 65536.0f;
+// Relative separation below which two fp64 gaps count as a near-tie (about
+// 64 ulp of the sum of the four u values involved).
+constexpr double kTieRel = 1.0 / 281474976710656.0;  // 2^-48
 
 struct SchedShared {
   int slot[kMaxEntries];
@@ -50,6 +54,7 @@ struct SchedShared {
   int ref[kMaxEntries][kMaxPassFrames + 1];
   float w[kMaxEntries][kMaxPassFrames + 1];
   float u32[kMaxEntries];
+  double u64[kMaxEntries];   // fp64 u at the endpoints of the candidate pairs
   int dest[kMaxEntries];     // plan: destination index of a changed entry, -1 if unchanged
   int src0[kMaxEntries];     // plan: first source index of a changed entry
 };
@@ -81,7 +86,7 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
   int count = mi.count;
   if (count != expected_count || count < 0 || count > M) {
     if (lane == 0) atomicOr(status, kStatusCountMismatch);
-    if (lane == 0) out->plan.n_src = 0;
+    if (lane == 0) { out->plan.n_src = 0; out->plan.near_tie_t = -1; }
     return;
   }
   const long long t0 = mi.t_next;
@@ -97,6 +102,7 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
   }
   __syncwarp();
   int merged[kMaxPassFrames];
+  long long near_tie = -1;  // first frame of the pass decided on a near-tie (lane 0)
   for (int f = 0; f < frames; ++f) {
     const long long t = t0 + f;
     if (lane == 0) {  // Append (K_t, V_t, t, 1)
@@ -124,8 +130,8 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) ub = fminf(ub, __shfl_xor_sync(0xffffffffu, ub, off));
-    double best = INFINITY;
-    int bi = 0x7fffffff, ncand = 0;
+    // Candidates: pairs whose fp32 interval reaches ub (npairs < 64: one bit each).
+    unsigned long long cm = 0;
     for (int i0 = 0; i0 < npairs; i0 += 32) {
       const int i = i0 + lane;
       bool cand = false;
@@ -133,24 +139,63 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
         const float a = s.u32[i], b = s.u32[i + 1];
         cand = fabsf(b - a) - kU32RelErr * (a + b) <= ub;
       }
-      const unsigned mask = __ballot_sync(0xffffffffu, cand);
-      ncand += __popc(mask);
-      if (cand && i < bi) bi = i;  // lowest-index candidate of this lane
+      cm |= (unsigned long long)__ballot_sync(0xffffffffu, cand) << i0;
     }
-    if (ncand > 1) {  // several pairs may be the minimum: decide in fp64
-      bi = 0x7fffffff;
-      for (int i = lane; i < npairs; i += 32) {
-        const float a = s.u32[i], b = s.u32[i + 1];
-        if (fabsf(b - a) - kU32RelErr * (a + b) <= ub) {
-          const double g = fabs(warp_u(0.5 * (double)(2 * t - s.mu2[i + 1]), beta) -
-                                warp_u(0.5 * (double)(2 * t - s.mu2[i]), beta));
-          if (g < best) { best = g; bi = i; }
+    if (cm == 0) cm = (1ull << npairs) - 1;  // no finite bound (cannot happen for finite u): decide all in fp64
+    int bi;
+    if (__popcll(cm) == 1) {
+      bi = __ffsll((long long)cm) - 1;  // the single candidate
+    } else {
+      // Several pairs may be the minimum: decide in fp64.  u is evaluated once
+      // per endpoint of a candidate pair, one endpoint per lane (fp64 is slow
+      // on this part, so the evaluations run side by side, not per pair).
+      const unsigned long long em = cm | (cm << 1);
+      const int nep = __popcll(em);
+      for (int r0 = 0; r0 < nep; r0 += 32) {
+        const int r = r0 + lane;
+        if (r < nep) {
+          unsigned long long m = em;
+          for (int k = 0; k < r; ++k) m &= m - 1;  // drop the r lowest endpoints
+          const int e = __ffsll((long long)m) - 1;
+          s.u64[e] = warp_u(0.5 * (double)(2 * t - s.mu2[e]), beta);
         }
       }
+      __syncwarp();
+      double best = INFINITY;
+      bi = 0x7fffffff;
+      for (int i = lane; i < npairs; i += 32)
+        if ((cm >> i) & 1) {
+          const double g = fabs(s.u64[i + 1] - s.u64[i]);
+          if (g < best) { best = g; bi = i; }
+        }
       warp_argmin(best, bi);
-    } else {
-      double v = 0.0;
-      warp_argmin(v, bi);  // the single candidate
+      double second = INFINITY;
+      int si = 0x7fffffff;
+      for (int i = lane; i < npairs; i += 32)
+        if (((cm >> i) & 1) && i != bi) {
+          const double g = fabs(s.u64[i + 1] - s.u64[i]);
+          if (g < second) { second = g; si = i; }
+        }
+      warp_argmin(second, si);
+      // Certify the decision.  Any faithful fp64 d^beta (this one, or a host
+      // libm's) is within a few ulp of the true value, so two gaps closer than
+      // 2^-48 (u_b + u_b+1 + u_s + u_s+1) may be ordered differently by another
+      // evaluation.  Exact evaluations settle every comparison the same way:
+      // beta = 1 (u(d) = d) and beta = 0.5 where every u involved is an exact
+      // square root.
+      if (lane == 0 && si != 0x7fffffff) {
+        const double ub0 = s.u64[bi], ub1 = s.u64[bi + 1], us0 = s.u64[si], us1 = s.u64[si + 1];
+        bool exact = beta == 1.0;
+        if (beta == 0.5) {
+          exact = true;
+          const int ix[4] = {bi, bi + 1, si, si + 1};
+          for (int k = 0; k < 4; ++k) {
+            const double u = s.u64[ix[k]];
+            exact = exact && fma(u, u, -0.5 * (double)(2 * t - s.mu2[ix[k]])) == 0.0;
+          }
+        }
+        if (!exact && second - best <= kTieRel * (ub0 + ub1 + us0 + us1) && near_tie < 0) near_tie = t;
+      }
     }
     const int j = bi;
     merged[f] = j;
@@ -264,6 +309,7 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
     p.n_dest = nd;
     p.frames = frames;
     p.op = op;
+    p.near_tie_t = near_tie;
     for (int f = 0; f < kMaxPassFrames; ++f) p.merged_pair[f] = f < frames ? merged[f] : -1;
     m.count = count;
     m.t_next = t0 + frames;
@@ -452,6 +498,14 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS, kRope)) 
       if (blockIdx.x == 1) {
         atomicAdd(&a.totals[0], (unsigned long long)(p.n_src + p.n_dest));  // per layer, K and V
         atomicAdd(&a.totals[1], 1ull);
+        // A decision of this pass that the schedule could not certify: report
+        // it (first frame kept) now that the pass is applied.
+        const long long nt = p.near_tie_t;
+        if (nt >= 0) {
+          atomicOr(a.status, kStatusNearTie);
+          atomicCAS(reinterpret_cast<unsigned long long*>(reinterpret_cast<char*>(a.status) + kNearTieFrameOffset),
+                    0ull, (unsigned long long)(nt + 1));
+        }
       }
     }
   }
@@ -549,13 +603,7 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   const int nvec = g.N * dv;
   // One wave: (SMs x resident blocks) spread evenly over the layer*K|V*head rows;
   // each thread then strides over its row's vectors.
-  static int num_sms = 0;
-  if (num_sms == 0) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) !=
-                                                   cudaSuccess)
-      num_sms = 148;
-  }
+  const int num_sms = current_device_sm_count(148);
   const int nsb = frames <= 2 ? 0 : frames == 3 ? 1 : 2;  // sources <= 3F: 6, 9 or 12
   const int rows = g.L * 2 * g.H;
   int bx = (num_sms * cons_blocks_per_sm(6 + 3 * nsb, rope.pairs > 0) - 1) / rows;  // - 1: the lookahead block
@@ -671,13 +719,7 @@ cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* 
   int dv = g.D / per_vec, shift = 0;
   while ((1 << shift) < dv) ++shift;
   a.dv_shift = shift;
-  static int num_sms = 0;
-  if (num_sms == 0) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev) !=
-                                                   cudaSuccess)
-      num_sms = 148;
-  }
+  const int num_sms = current_device_sm_count(148);
   const long long rows = (long long)g.L * g.H * count;
   const int nvec = g.N * dv;
   long long bx = (long long)num_sms * 8 / rows;  // one wave of 8 resident blocks per SM
@@ -691,6 +733,16 @@ cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* 
   else
     rephase_kernel<float><<<grid, 256, 0, stream>>>(a);
   return cudaGetLastError();
+}
+
+int current_device_sm_count(int fallback) {
+  static PerDevice<int> table;
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return fallback;
+  const bool ok = table.get(dev, [](int d, int* v) {
+    return cudaDeviceGetAttribute(v, cudaDevAttrMultiProcessorCount, d) == cudaSuccess && *v > 0;
+  }, &n);
+  return ok ? n : fallback;
 }
 
 }  // namespace fademem

@@ -13,6 +13,7 @@
 #include <nvtx3/nvToolsExt.h>
 
 #include "fademem_internal.h"
+#include "per_device.h"
 
 using namespace fademem;
 
@@ -454,11 +455,25 @@ FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void* stream_,
   unsigned int w = 0;
   e = cudaMemcpy(&w, h->status, sizeof(w), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "reading the device status");
+  unsigned long long tie = 0;  // frame + 1 of the first uncertified schedule decision
+  char* tie_slot = reinterpret_cast<char*>(h->status) + kNearTieFrameOffset;
+  if (w & kStatusNearTie) {
+    e = cudaMemcpy(&tie, tie_slot, sizeof(tie), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device status");
+  }
   const unsigned int zero = 0;
   e = cudaMemcpy(h->status, &zero, sizeof(zero), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
+  const unsigned long long zero64 = 0;
+  e = cudaMemcpy(tie_slot, &zero64, sizeof(zero64), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the device status");
   if (word) *word = w;
   if (w & kStatusTimeout) return fail(FADEMEM_ERR_DEVICE_TIMEOUT, "a device wait timed out (status 0x%x)", w);
+  if (w & kStatusNearTie)
+    return fail(FADEMEM_ERR_DEVICE_CHECK,
+                "%sschedule decision at frame %lld not certified: its two smallest warped gaps are equal within "
+                "the fp64 evaluation error of d^beta (status 0x%x)",
+                w != kStatusNearTie ? "a device check failed; " : "", (long long)tie - 1, w);
   if (w) return fail(FADEMEM_ERR_DEVICE_CHECK, "a device check failed (status 0x%x)", w);
   return FADEMEM_OK;
 }
@@ -502,25 +517,26 @@ namespace {
 // kernel: on the host it is only a stand-in; its device address comes from
 // cudaGetSymbolAddress, once per device.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[FADEMEM_NOALLOC_SCRATCH_BYTES];
+// DevState holds the entry table of the largest budget fademem_create accepts
+// (kMaxEntries = FADEMEM_MAX_BUDGET + 1), so every handle's state fits.
 static_assert(sizeof(DevState) <= FADEMEM_NOALLOC_SCRATCH_BYTES, "DevState must fit the no-alloc scratch");
+static_assert(kMaxEntries == FADEMEM_MAX_BUDGET + 1, "the entry table must hold every budget fademem_create accepts");
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+PerDevice<void*> g_scratch_addr;
 
 fademem_status noalloc_scratch(DevState** out) {
   int dev = -1;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  if (dev < 0 || dev >= kMaxDevices) return fail(FADEMEM_ERR_UNSUPPORTED, "device %d out of range", dev);
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // with this device current
-    if (e != cudaSuccess) return cuda_fail(e, "looking up the no-alloc scratch");
-    g_scratch_addr[dev] = p;
-  }
-  *out = reinterpret_cast<DevState*>(g_scratch_addr[dev]);
+  cudaError_t lookup = cudaSuccess;
+  void* p = nullptr;
+  const bool ok = g_scratch_addr.get(dev, [&lookup](int, void** v) {
+    lookup = cudaGetSymbolAddress(v, g_noalloc_scratch);  // with this device current
+    return lookup == cudaSuccess;
+  }, &p);
+  if (!ok && lookup != cudaSuccess) return cuda_fail(lookup, "looking up the no-alloc scratch");
+  if (!ok) return fail(FADEMEM_ERR_UNSUPPORTED, "device %d out of range", dev);
+  *out = reinterpret_cast<DevState*>(p);
   return FADEMEM_OK;
 }
 
@@ -532,9 +548,6 @@ FADEMEM_API fademem_status fademem_consolidate_noalloc(fademem_t h, void* stream
   NvtxRange nvtx_("fademem_consolidate_noalloc");
   if (!h) return fail(FADEMEM_ERR_INVALID_ARG, "handle is NULL");
   h->chained = false;
-  if (h->g.M + 1 > kMaxEntries)
-    return fail(FADEMEM_ERR_UNSUPPORTED, "budget %d does not fit the %d-byte no-alloc scratch", h->g.M,
-                FADEMEM_NOALLOC_SCRATCH_BYTES);
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   DevState* scratch = nullptr;
   fademem_status s = noalloc_scratch(&scratch);

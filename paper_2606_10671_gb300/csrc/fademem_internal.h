@@ -18,9 +18,15 @@ constexpr int kMaxEntries = FADEMEM_MAX_BUDGET + 1;
 constexpr int kMaxRopePairs = 64;  // head_dim / 2 at head_dim 128
 
 // Device status word bits (fademem_get_device_status).
-constexpr uint32_t kStatusTimeout = 1u << 0;      // a bounded mbarrier wait gave up
-constexpr uint32_t kStatusCountMismatch = 1u << 1;  // host and device entry counts disagree
-constexpr uint32_t kStatusPlanOverflow = 1u << 2;  // merge plan exceeded its static bounds
+constexpr uint32_t kStatusTimeout = FADEMEM_STATUS_TIMEOUT;              // a bounded mbarrier wait gave up
+constexpr uint32_t kStatusCountMismatch = FADEMEM_STATUS_COUNT_MISMATCH;  // host and device entry counts disagree
+constexpr uint32_t kStatusPlanOverflow = FADEMEM_STATUS_PLAN_OVERFLOW;    // merge plan exceeded its static bounds
+// A schedule decision whose best and second-best warped gaps lie within the
+// fp64 evaluation error of each other (and are not exact): another correct fp64
+// evaluation of u(d) = d^beta could pick the other pair.  The frame of the first
+// such decision is kept at byte kNearTieFrameOffset of the workspace (frame + 1).
+constexpr uint32_t kStatusNearTie = FADEMEM_STATUS_NEAR_TIE;
+constexpr size_t kNearTieFrameOffset = 24;  // after the status word and the two counters
 
 // Entry table of the memory (Sec. 3.3 "memory entries"), temporal order.
 struct DevMeta {
@@ -48,6 +54,7 @@ struct DevPlan {
   int src_dest[kMaxSrc];
   int dest_slot[kMaxDest];
   int merged_pair[kMaxPassFrames];   // j chosen for each frame (-1: no merge)
+  long long near_tie_t;              // first frame of the pass decided on a near-tie, -1 if none
 };
 
 struct DevState {
@@ -117,6 +124,10 @@ cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc,
 cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
                                const void* Vcur, int Lk2, const void* Q, void* out, int Lq, float scale,
                                unsigned int* status, cudaStream_t stream, char* err, size_t errlen);
+
+// Multiprocessor count of the current device, looked up once per device
+// (PerDevice table, thread-safe); `fallback` if the query fails.
+int current_device_sm_count(int fallback);
 
 // Waits on an mbarrier that is never signalled, through the same bounded wait
 // the kernels use; sets kStatusTimeout after limit_cycles.

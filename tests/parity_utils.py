@@ -75,6 +75,7 @@ class Pair:
         self.anchor = anchor
         self.input_max = 0.0
         self.rounds = {}
+        self.margins = []  # the oracle's relative margin of every decision, frame by frame
 
     def _frames(self, gen, n):
         if self.device_gen:
@@ -101,6 +102,8 @@ class Pair:
             self.input_max = max(self.input_max, float(np.abs(Kt).max()), float(np.abs(Vt).max()))
             for f in range(frames):
                 self.ora[l].insert(Kt[f], Vt[f])
+                if l == self.ora_layers[0]:
+                    self.margins.append(self.ora[l].last_margin)
 
     def step(self, frames: int = 3, per_call: int | None = None):
         before = self._spans()
@@ -214,3 +217,42 @@ class Pair:
         Qt = Qh[:, self.tracked, :]
         ref = self.ora[layer].attend(Qt, self.N, len(self.tracked), self.D)
         return assert_close(og[:, self.tracked, :], ref, self.dtype, "attention")
+
+
+class RoundingDepth:
+    """Bookkeeping of bf16 storage rounding per memory entry, keyed by (first, span).
+
+    r: the number of consolidation passes that rewrote (and so rounded) the entry's
+    block along its history (its deepest chain of merges); copies of new frames and
+    the anchor have r = 0.  a: the largest |input| over the entry's own source frames,
+    per coordinate.  Merges are convex and elementwise, so the exact block and every
+    rounded intermediate lie within +-a, and |stored - exact| <= r (2^-8 + 2^-20) a.
+    """
+
+    def __init__(self, anchor: bool = True):
+        self.anchor = anchor
+        self.r = {}
+        self.a = {}
+        self.anchor_a = None
+
+    def update(self, before, frames_before, fresh, after, passes: int = 1):
+        """One consolidate call: `before`/`after` the (first, span) lists of the entries,
+        `fresh` {frame: |values|} of the frames it inserted, `passes` fused passes."""
+        if 0 in fresh:
+            self.anchor_a = fresh[0]
+        old = set(before)
+        r, a = {}, {}
+        for key in after:
+            f, s = key
+            if key in old:
+                r[key], a[key] = self.r[key], self.a[key]
+            elif f == 0 and self.anchor:
+                r[key], a[key] = 0, self.anchor_a
+            elif s == 1 and f >= frames_before:
+                r[key], a[key] = 0, fresh[f]
+            else:
+                inner = [k for k in self.r if k[0] >= f and k[0] + k[1] <= f + s]
+                parts = [self.a[k] for k in inner] + [x for g, x in fresh.items() if f <= g < f + s]
+                r[key] = passes + max([self.r[k] for k in inner], default=0)
+                a[key] = np.maximum.reduce(parts)
+        self.r, self.a = r, a

@@ -98,6 +98,49 @@ def test_beta_values(beta):
     p.check_memory()
 
 
+@pytest.mark.parametrize("per_call", [1, 3])
+def test_schedule_near_tie_is_flagged(per_call):
+    """Algorithm S1's argmin at beta = 1 - 2^-48.  Pairs whose gaps tie exactly at beta = 1
+    now differ by about 1e-15 relative, below the error of any fp64 evaluation of d^beta,
+    so no fp64 computation can certify which one is smaller.  The oracle (host libm pow)
+    shows these near-ties through its margin.  The device must decide every earlier frame
+    exactly as the oracle does and flag the first near-tie through its status word
+    (FADEMEM_STATUS_NEAR_TIE, the message naming the frame).  A certified exponent (0.3)
+    on the same call pattern leaves the word clear."""
+    import re
+    from oracle import OracleMemory
+    from paper_2606_10671_gb300 import FadeMem, capi
+    M, N, H, D, frames = 8, 4, 1, 64, 48
+    for beta, near_tie in ((1.0 - 2.0 ** -48, True), (0.3, False)):
+        mem = FadeMem(M, H, D, N, beta=beta, dtype=torch.float32)
+        ora = OracleMemory(M, beta, anchor=True)
+        X = torch.zeros((per_call * N, H, D), device="cuda")
+        margins, first = [], None
+        for f0 in range(0, frames, per_call):
+            mem.insert(0, X, X)
+            mem.consolidate()
+            for _ in range(per_call):
+                ora.insert()
+                margins.append(ora.last_margin)
+            if first is None and min(margins) < 1e-12:
+                first = next(f for f, m in enumerate(margins) if m < 1e-12)
+            if first is None:  # every decision so far certified: bit-exact
+                slot, fst, span, mu2 = mem.entries()
+                o_slot, o_first, o_span, o_mu = ora.entries()
+                assert (slot.tolist(), fst.tolist(), span.tolist()) == \
+                    (o_slot.tolist(), o_first.tolist(), o_span.tolist()), f0
+                assert mu2.tolist() == [int(round(2 * m)) for m in o_mu], f0
+        st, word = mem.device_status(raise_on_error=False)
+        msg = capi.load().fademem_last_error().decode()
+        if not near_tie:
+            assert first is None and (st, word) == (0, 0), (st, word, msg)
+            continue
+        assert first is not None and all(m > 1e-3 for m in margins[:first])
+        assert st == capi.FADEMEM_ERR_DEVICE_CHECK and word == capi.STATUS_NEAR_TIE, (st, word, msg)
+        assert int(re.search(r"frame (\d+)", msg).group(1)) == first, (msg, first)
+        assert mem.device_status() == (0, 0)  # read and cleared
+
+
 @pytest.mark.parametrize("per_call,frames", [(1, 3), (3, 3), (2, 7), (7, 7), (5, 13)])
 def test_insert_granularity(per_call, frames):
     """Frames inserted in several calls and consolidated together (passes of <= 4 frames,
@@ -472,6 +515,33 @@ def test_fuzz_small_configurations(case):
     p.check_attend(p.queries(c["Lq"], step=seg))
     Kc, Vc = p.chunk(c["ncur"], step=seg)
     p.check_attend_ext(p.queries(c["Lq"], step=seg + 1), Kc, Vc)
+    p.gpu.device_status()
+
+
+@pytest.mark.parametrize("case", range(16))
+def test_fuzz_arbitrary_beta(case):
+    """The fuzz above with beta drawn from (0.05, 1] instead of the certified set.  The
+    schedule's guarantee at any beta: every decision equals the oracle's, or the device
+    flags it (FADEMEM_STATUS_NEAR_TIE) and the oracle's own margin at that frame shows a
+    near-tie.  Checked after every segment: the entry table bit-exact while nothing is
+    flagged, and every stored block within tolerance."""
+    from paper_2606_10671_gb300 import capi
+    c = _fuzz_case(100 + case)
+    c["beta"] = float(np.random.default_rng([4343, case]).uniform(0.05, 1.0))
+    p = Pair(c["M"], c["H"], c["D"], c["N"], beta=c["beta"], anchor=c["anchor"], op=c["op"], dtype=c["dtype"],
+             seed=c["seed"], rope_pairs=c["rope"])
+    for seg in range(c["segments"]):
+        p.step(c["frames"], per_call=c["per_call"])
+        st, word = p.gpu.device_status(raise_on_error=False)
+        if word & capi.STATUS_NEAR_TIE:
+            import re
+            frame = int(re.search(r"frame (\d+)", capi.load().fademem_last_error().decode()).group(1))
+            assert p.margins[frame] < 1e-9, (frame, p.margins[frame])
+            return
+        assert (st, word) == (0, 0)
+        p.check_entries()
+        p.check_memory()
+    p.check_attend(p.queries(c["Lq"], step=seg))
     p.gpu.device_status()
 
 

@@ -76,3 +76,7 @@ def test_reference_arm_two_ranks_rank0_prints_once():
     line = json.loads(outs[0].splitlines()[-1])
     assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle"
+    sys.path.insert(0, ROOT)
+    import bench
+    assert line["config"] == bench.main_config(2)  # the same config object as the GPU arm's line
+    assert line["ms_per_step"] <= line["ms_per_step_extrapolated"]  # measured sample vs full-step estimate

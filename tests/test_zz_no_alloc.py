@@ -31,25 +31,38 @@ def _close(a: torch.Tensor, b: torch.Tensor, dtype):
     assert np.all(np.isfinite(a)) and err <= bound, (err, bound)
 
 
-@pytest.mark.parametrize("dtype,D", [(torch.bfloat16, 128), (torch.float32, 64)])
-def test_consolidate_noalloc_matches_consolidate(cuda_lib, dtype, D):
+# (dtype, head_dim, temporal RoPE pairs, frames of each insert call per segment).  A
+# call's frames split into fused passes of at most 4 that never cross an insert, so
+# (2, 4) and (5,) make two passes per consolidate; RoPE adds the re-phase kernel.
+CASES = [(torch.bfloat16, 128, 0, (3,)), (torch.float32, 64, 0, (3,)),
+         (torch.bfloat16, 128, 22, (3,)), (torch.float32, 64, 8, (2, 4)), (torch.bfloat16, 128, 0, (5,))]
+
+
+@pytest.mark.parametrize("dtype,D,rope,chunks", CASES)
+def test_consolidate_noalloc_matches_consolidate(cuda_lib, dtype, D, rope, chunks):
     from paper_2606_10671_gb300 import FadeMem, capi
     lib = capi.load(cuda_lib)
     M, H, N, L = 5, 3, 100, 2
-    ref = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=dtype)
-    new = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=dtype)
+    ref = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=dtype, rope_pairs=rope)
+    new = FadeMem(M, H, D, N, num_layers=L, beta=0.3, dtype=dtype, rope_pairs=rope)
     stream = torch.cuda.current_stream()
     sp = ctypes.c_void_p(int(stream.cuda_stream))
     gens = [(HostAR1((N, H, D), 3, KIND_K, l), HostAR1((N, H, D), 3, KIND_V, l)) for l in range(L)]
-    for seg in range(9):  # 27 frames through a 5-entry budget: merges in every call from the 2nd on
+    per_seg = sum(chunks)
+    for seg in range(9):  # 27+ frames through a 5-entry budget: merges in every call from the 2nd on
         keep = []
         for l, (gk, gv) in enumerate(gens):
-            K = torch.from_numpy(np.stack([gk.next() for _ in range(3)])).to(dtype).cuda()
-            V = torch.from_numpy(np.stack([gv.next() for _ in range(3)])).to(dtype).cuda()
+            K = torch.from_numpy(np.stack([gk.next() for _ in range(per_seg)])).to(dtype).cuda()
+            V = torch.from_numpy(np.stack([gv.next() for _ in range(per_seg)])).to(dtype).cuda()
             keep.append((K, V))
-            for mem in (ref, new):
-                assert lib.fademem_insert(ctypes.c_void_p(mem.handle), l, ctypes.c_void_p(K.data_ptr()),
-                                          ctypes.c_void_p(V.data_ptr()), 3) == capi.FADEMEM_OK
+            a = 0
+            for n in chunks:
+                Kc, Vc = K[a:a + n].contiguous(), V[a:a + n].contiguous()
+                keep.append((Kc, Vc))
+                a += n
+                for mem in (ref, new):
+                    assert lib.fademem_insert(ctypes.c_void_p(mem.handle), l, ctypes.c_void_p(Kc.data_ptr()),
+                                              ctypes.c_void_p(Vc.data_ptr()), n) == capi.FADEMEM_OK
         assert lib.fademem_consolidate(ctypes.c_void_p(ref.handle), sp) == capi.FADEMEM_OK
         st = lib.fademem_consolidate_noalloc(ctypes.c_void_p(new.handle), sp)
         assert st == capi.FADEMEM_OK, capi.fademem_last_error()
@@ -62,6 +75,10 @@ def test_consolidate_noalloc_matches_consolidate(cuda_lib, dtype, D):
         for l in range(L):
             for x, y in zip(new.layer_memory(l), ref.layer_memory(l)):
                 _close(x[:, :count], y[:, :count], dtype)  # occupied slots only
+        if seg == 0:
+            b0 = new.stats()[1]
+        elif seg == 1:
+            assert new.stats()[1] - b0 == len(chunks) + (1 if chunks == (5,) else 0)  # passes per call
         Q = torch.from_numpy(host_queries((150, H, D), 3, 0, seg)).to(dtype).cuda()
         for l in range(L):
             _close(new.attend(l, Q), ref.attend(l, Q), dtype)
