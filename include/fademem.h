@@ -53,6 +53,10 @@ extern "C" {
 #define FADEMEM_STATUS_COUNT_MISMATCH 0x2u
 #define FADEMEM_STATUS_PLAN_OVERFLOW 0x4u
 #define FADEMEM_STATUS_NEAR_TIE 0x8u
+#define FADEMEM_STATUS_BOUNDS 0x10u
+
+/* Bits of fademem_build_flags(). */
+#define FADEMEM_BUILD_DEBUG_BOUNDS 0x1u
 
 typedef enum fademem_status {
     FADEMEM_OK = 0,
@@ -216,7 +220,11 @@ FADEMEM_API fademem_status fademem_layer_memory(fademem_t h, int layer, void **K
  *     but another fp64 evaluation of d^beta, such as a host libm's, may
  *     choose the other pair.  The message names the first such frame.
  * Every other configuration decides each merge exactly as an fp64 evaluation
- * of Algorithm S1 does. */
+ * of Algorithm S1 does.
+ *   FADEMEM_STATUS_BOUNDS          (bounds-checking build only, see
+ *     fademem_build_flags) a kernel found a global-memory access outside the
+ *     buffer it belongs to, or a table index outside its array, and skipped
+ *     it; the results of that call are not to be trusted. */
 FADEMEM_API fademem_status fademem_get_device_status(fademem_t h, void *stream, uint32_t *word);
 
 /* Diagnostic of device-side failure detection: enqueues one thread that waits,
@@ -311,6 +319,16 @@ FADEMEM_API fademem_status fademem_import_state(fademem_t h, const void *host_bu
 
 /* Release the handle (NULL-safe).  Does not free the caller's workspace. */
 FADEMEM_API void fademem_destroy(fademem_t h);
+
+/* How this library was built (no counterpart in the paper): a set of
+ * FADEMEM_BUILD_* bits.  FADEMEM_BUILD_DEBUG_BOUNDS: every kernel checks each
+ * global-memory access against the buffer it belongs to (the workspace's
+ * memory slabs, the caller's frames, queries and outputs) and each table
+ * index against its array, skips an access that fails and sets
+ * FADEMEM_STATUS_BOUNDS; built by `build.py --debug-bounds` as
+ * libfademem_debug.so, slower, for testing.  0 for the release library.
+ * Needs no GPU. */
+FADEMEM_API uint32_t fademem_build_flags(void);
 
 /* Message of the last failed call on this thread ("" if none). */
 FADEMEM_API const char *fademem_last_error(void);

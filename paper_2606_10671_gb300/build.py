@@ -4,6 +4,11 @@ Each translation unit under csrc/ compiles in parallel to an object in
 _build/, then nvcc links them with the static CUDA runtime, so the library
 loads on a machine without a driver (for the symbol checks) and needs no
 libcudart at run time.  A source hash skips rebuilds when nothing changed.
+
+`--debug-bounds` (build_library(debug_bounds=True)) builds
+libfademem_debug.so instead, with -DFADEMEM_DEBUG_BOUNDS: every kernel then
+checks each global-memory access and table index and reports a failure
+through the device status word (FADEMEM_STATUS_BOUNDS) rather than making it.
 """
 from __future__ import annotations
 
@@ -19,6 +24,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfademem.so")
+LIB_DEBUG = os.path.join(HERE, "libfademem_debug.so")
+DEBUG_FLAGS = ["-DFADEMEM_DEBUG_BOUNDS"]
 INCLUDE = os.path.join(ROOT, "include")
 SOURCES = ["fademem_api.cu", "consolidate.cu", "attend_simt.cu", "attend_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -32,7 +39,7 @@ def _nvcc() -> str:
     return cand
 
 
-def _digest() -> str:
+def _digest(extra: list[str]) -> str:
     h = hashlib.sha256()
     files = sorted(os.listdir(CSRC)) + ["../../include/fademem.h", "../build.py"]
     for name in files:
@@ -41,24 +48,28 @@ def _digest() -> str:
             h.update(name.encode())
             with open(path, "rb") as fh:
                 h.update(fh.read())
-    h.update(" ".join(ARCH + NVCC_FLAGS).encode())
+    h.update(" ".join(ARCH + NVCC_FLAGS + extra).encode())
     return h.hexdigest()
 
 
-def build_library(force: bool = False, verbose: bool = False) -> str:
-    """Compile (if stale) and return the path of libfademem.so."""
-    stamp = os.path.join(BUILD, "stamp")
-    digest = _digest()
-    if not force and os.path.exists(LIB) and os.path.exists(stamp):
+def build_library(force: bool = False, verbose: bool = False, debug_bounds: bool = False) -> str:
+    """Compile (if stale) and return the path of libfademem.so (libfademem_debug.so
+    with device bounds checks when debug_bounds)."""
+    extra = DEBUG_FLAGS if debug_bounds else []
+    out = LIB_DEBUG if debug_bounds else LIB
+    build = os.path.join(BUILD, "debug") if debug_bounds else BUILD
+    stamp = os.path.join(build, "stamp")
+    digest = _digest(extra)
+    if not force and os.path.exists(out) and os.path.exists(stamp):
         with open(stamp) as fh:
             if fh.read().strip() == digest:
-                return LIB
-    os.makedirs(BUILD, exist_ok=True)
+                return out
+    os.makedirs(build, exist_ok=True)
     nvcc = _nvcc()
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
-        cmd = [nvcc, *ARCH, *NVCC_FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+        obj = os.path.join(build, src.replace(".cu", ".o"))
+        cmd = [nvcc, *ARCH, *NVCC_FLAGS, *extra, "-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             cmd.insert(1, "-Xptxas=-v")
         r = subprocess.run(cmd, capture_output=True, text=True)
@@ -70,16 +81,17 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = out + f".tmp{os.getpid()}"
     cmd = [nvcc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs, "-ldl"]  # -ldl: NVTX loads its tool lazily
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    os.replace(tmp, out)
     with open(stamp, "w") as fh:
         fh.write(digest)
-    return LIB
+    return out
 
 
 if __name__ == "__main__":
-    print(build_library(force="--force" in sys.argv, verbose="-v" in sys.argv))
+    print(build_library(force="--force" in sys.argv, verbose="-v" in sys.argv,
+                        debug_bounds="--debug-bounds" in sys.argv))

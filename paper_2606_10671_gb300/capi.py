@@ -26,6 +26,9 @@ STATUS_TIMEOUT = 0x1
 STATUS_COUNT_MISMATCH = 0x2
 STATUS_PLAN_OVERFLOW = 0x4
 STATUS_NEAR_TIE = 0x8
+STATUS_BOUNDS = 0x10
+# Bits of fademem_build_flags() (FADEMEM_BUILD_*).
+BUILD_DEBUG_BOUNDS = 0x1
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "WORKSPACE", 4: "EMPTY", 5: "PENDING", 6: "CUDA",
                 7: "DEVICE_TIMEOUT", 8: "DEVICE_CHECK"}
 
@@ -42,7 +45,7 @@ EXPORTS = ("fademem_workspace_bytes", "fademem_create", "fademem_insert", "fadem
            "fademem_layer_memory", "fademem_get_device_status",
            "fademem_selftest_wait_timeout", "fademem_reset", "fademem_consolidate_noalloc",
            "fademem_host_staging_bytes", "fademem_step_host", "fademem_state_bytes", "fademem_export_state",
-           "fademem_import_state", "fademem_destroy", "fademem_last_error")
+           "fademem_import_state", "fademem_destroy", "fademem_build_flags", "fademem_last_error")
 
 
 class fademem_config(ctypes.Structure):
@@ -98,6 +101,7 @@ def load(path: str | None = None):
             "fademem_export_state": (I, [P, P, ctypes.c_size_t, P]),
             "fademem_import_state": (I, [P, P, ctypes.c_size_t, P]),
             "fademem_destroy": (None, [P]),
+            "fademem_build_flags": (ctypes.c_uint32, []),
             "fademem_last_error": (ctypes.c_char_p, []),
         }
         for name, (res, args) in sig.items():

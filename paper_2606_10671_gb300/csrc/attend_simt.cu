@@ -17,13 +17,20 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
                                                          int Lk, const float* __restrict__ Kcur,
                                                          const float* __restrict__ Vcur, int Lk2,
                                                          const float* __restrict__ Q, float* __restrict__ out,
-                                                         int Lq, int H, size_t head_stride, float scale_log2) {
+                                                         int Lq, int H, size_t head_stride, float scale_log2,
+                                                         unsigned int* status) {
   constexpr int P = D / 32;
   const int lane = threadIdx.x & 31;
   const long long gw = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   if (gw >= (long long)Lq * H) return;
   const int q = (int)(gw / H), h = (int)(gw % H);
   const float* qp = Q + ((size_t)q * H + h) * D;
+  // Buffers for the bounds-checking build: the layer's K and V memory, the
+  // chunk's K and V, Q and out.
+  const DevRange k_r = dev_range(Kc, (size_t)H * head_stride * 4), v_r = dev_range(Vc, (size_t)H * head_stride * 4);
+  const DevRange kc_r = dev_range(Kcur, (size_t)Lk2 * H * D * 4), vc_r = dev_range(Vcur, (size_t)Lk2 * H * D * 4);
+  const DevRange q_r = dev_range(Q, (size_t)Lq * H * D * 4), o_r = dev_range(out, (size_t)Lq * H * D * 4);
+  if (kBoundsChecks && !bounds_ok(q_r, qp, D * 4, status)) return;
   float qv[P], o[P];
 #pragma unroll
   for (int i = 0; i < P; ++i) { qv[i] = qp[lane + 32 * i]; o[i] = 0.f; }
@@ -33,6 +40,9 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
   for (int k = 0; k < Lk + Lk2; ++k) {
     const float* kr = k < Lk ? Kh + (size_t)k * D : Kcur + ((size_t)(k - Lk) * H + h) * D;
     const float* vr = k < Lk ? Vh + (size_t)k * D : Vcur + ((size_t)(k - Lk) * H + h) * D;
+    if (kBoundsChecks &&
+        (!bounds_ok(k < Lk ? k_r : kc_r, kr, D * 4, status) || !bounds_ok(k < Lk ? v_r : vc_r, vr, D * 4, status)))
+      continue;
     float dot = 0.f;
 #pragma unroll
     for (int i = 0; i < P; ++i) dot = fmaf(qv[i], kr[lane + 32 * i], dot);
@@ -48,6 +58,7 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
     m = m_new;
   }
   float* op = out + ((size_t)q * H + h) * D;
+  if (kBoundsChecks && !bounds_ok(o_r, op, D * 4, status)) return;
   const float inv = 1.f / l;
 #pragma unroll
   for (int i = 0; i < P; ++i) op[lane + 32 * i] = o[i] * inv;
@@ -57,7 +68,7 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
 
 cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
                               const void* Vcur, int Lk2, const float* Q, float* out, int Lq, float scale,
-                              cudaStream_t stream) {
+                              unsigned int* status, cudaStream_t stream) {
   const long long warps = (long long)Lq * g.H;
   const int threads = 256;
   const long long blocks = (warps * 32 + threads - 1) / threads;
@@ -66,11 +77,11 @@ cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc,
   if (g.D == 128)
     attend_f32_kernel<128><<<(unsigned)blocks, threads, 0, stream>>>(
         (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
-        head_stride, scale_log2);
+        head_stride, scale_log2, status);
   else
     attend_f32_kernel<64><<<(unsigned)blocks, threads, 0, stream>>>(
         (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
-        head_stride, scale_log2);
+        head_stride, scale_log2, status);
   return cudaGetLastError();
 }
 

@@ -295,6 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q0 = blockIdx.x * kBM;
   const int h = blockIdx.y;
+  if (kBoundsChecks && threadIdx.x == 0) index_ok(h, p.H, p.status);
   // Key tiles 0..n1-1 come from the memory, n1..n1+n2-1 from the current chunk.
   const int n1 = (p.Lk + kBN - 1) / kBN;
   const int n_tiles = n1 + (p.Lk2 + kBN - 1) / kBN;
@@ -357,6 +358,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
           break;
         }
         const uint32_t sK = sbase + kOffK + s * kTileBytes;
+        if (kBoundsChecks && !index_ok(j < n1 ? (long long)j * kBN : (long long)(j - n1) * kBN, j < n1 ? p.Lk : p.Lk2,
+                                       p.status)) {
+          *abort_flag = 1;  // stop the CTA: every role's waits give up on the abort flag
+          break;
+        }
         mbar_expect_tx(full, kTileBytes);
         if (j < n1) {
           tma_load_3d(sK, &p.tmK, full, 0, j * kBN, h);
@@ -590,7 +596,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
               v.y = pack_bf16(o[2], o[3]);
               v.z = pack_bf16(o[4], o[5]);
               v.w = pack_bf16(o[6], o[7]);
-              *reinterpret_cast<uint4*>(orow + col + i) = v;
+              if (!kBoundsChecks || bounds_ok(dev_range(p.out, (size_t)p.Lq * p.H * kHD * 2), orow + col + i,
+                                              sizeof(uint4), p.status))
+                *reinterpret_cast<uint4*>(orow + col + i) = v;
             }
           }
         }

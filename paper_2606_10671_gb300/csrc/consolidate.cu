@@ -117,6 +117,7 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
     count += 1;
     __syncwarp();
     merged[f] = -1;
+    if (kBoundsChecks && !index_ok(count - 1, kMaxEntries, status)) break;  // the append above stayed in the table
     if (count <= M) continue;
 
     // Eligible pairs: (i, i+1) for i <= count-3 (the pair holding the newest is excluded).
@@ -198,6 +199,7 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
       }
     }
     const int j = bi;
+    if (kBoundsChecks && !index_ok(j, count - 2, status)) break;  // an eligible pair: j + 1 <= count - 2
     merged[f] = j;
     if (lane == 0) {
       const long long sa = s.span[j], sb = s.span[j + 1];
@@ -294,9 +296,11 @@ __device__ __noinline__ void schedule_pass(SchedShared& s, const DevState* in, D
     for (int i = lane; i < count; i += 32) {
       const int d = s.dest[i];
       if (d < 0) continue;
+      if (kBoundsChecks && !index_ok(d, kMaxDest, status)) continue;
       p.dest_slot[d] = s.slot[i];
       for (int k = 0; k < s.natoms[i]; ++k) {
         const int q = s.src0[i] + k;
+        if (kBoundsChecks && !index_ok(q, kMaxSrc, status)) break;
         p.src_ref[q] = s.ref[i][k];
         p.src_w[q] = s.w[i][k];
         p.src_dest[q] = d;
@@ -368,6 +372,8 @@ template <> struct Vec<__nv_bfloat16> {
 
 struct ConsolidateArgs {
   char* cache;            // workspace cache base
+  size_t cache_bytes;     // every layer's memory, from cache (bounds checks)
+  size_t frame_bytes;     // one layer's K (or V) frames of the pass (bounds checks)
   const DevState* st;
   int L, H, M, N, D;
   int dv_shift;           // log2(D / elements per vector)
@@ -538,8 +544,17 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS, kRope)) 
     uint4 raw[kNS];
 #pragma unroll
     for (int k = 0; k < kNS; ++k)
-      if (k < ns)
-        raw[k] = __ldcs(reinterpret_cast<const uint4*>(s_base[k] + ((fmask >> k) & 1 ? off_frame : off_slab)));
+      if (k < ns) {
+        const bool fr = (fmask >> k) & 1;
+        const T* src = s_base[k] + (fr ? off_frame : off_slab);
+        if (kBoundsChecks && !bounds_ok(fr ? dev_range(a.srcs.src[l][kv], a.frame_bytes)
+                                           : dev_range(a.cache, a.cache_bytes),
+                                        src, sizeof(uint4), a.status)) {
+          raw[k] = make_uint4(0u, 0u, 0u, 0u);
+          continue;
+        }
+        raw[k] = __ldcs(reinterpret_cast<const uint4*>(src));
+      }
     float acc[V::kN];
 #pragma unroll
     for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? -INFINITY : 0.f;
@@ -554,7 +569,9 @@ __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS, kRope)) 
 #pragma unroll
         for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? fmaxf(acc[e], x[e]) : fmaf(w, x[e], acc[e]);
         if ((emask >> k) & 1) {
-          *reinterpret_cast<uint4*>(s_dst[k] + off_slab) = V::pack(acc);
+          T* dst = s_dst[k] + off_slab;
+          if (!kBoundsChecks || bounds_ok(dev_range(a.cache, a.cache_bytes), dst, sizeof(uint4), a.status))
+            *reinterpret_cast<uint4*>(dst) = V::pack(acc);
 #pragma unroll
           for (int e = 0; e < V::kN; ++e) acc[e] = kMax ? -INFINITY : 0.f;
         }
@@ -590,6 +607,8 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   a.rope_t0 = rope.t0;
   for (int k = 0; k < kMaxRopePairs; ++k) a.rope_omega[k] = rope.omega[k];
   a.cache = reinterpret_cast<char*>(cache_base);
+  a.cache_bytes = (size_t)g.L * g.layer_bytes;
+  a.frame_bytes = (size_t)frames * g.N * g.H * g.D * g.elem;
   a.st = st;
   a.L = g.L; a.H = g.H; a.M = g.M; a.N = g.N; a.D = g.D;
   const int per_vec = g.dtype == FADEMEM_BF16 ? 8 : 4;
@@ -642,6 +661,8 @@ namespace {
 
 struct RephaseArgs {
   char* cache;
+  size_t cache_bytes;  // every layer's memory, from cache (bounds checks)
+  unsigned int* status;
   const DevState* st;
   int H, M, N, D, count, bx, dv_shift, pairs;
   long long t_next;
@@ -664,7 +685,10 @@ __global__ void __launch_bounds__(256) rephase_kernel(const __grid_constant__ Re
   const int h = (row / a.count) % a.H;
   const int l = row / (a.count * a.H);
   int slot = a.st->meta.slot[i];
-  if (slot < 0 || slot >= a.M) return;  // not a valid table (refused earlier by the schedule checks)
+  if (slot < 0 || slot >= a.M) {  // not a valid table (refused earlier by the schedule checks)
+    if (kBoundsChecks && threadIdx.x == 0) atomicOr(a.status, kStatusBounds);
+    return;
+  }
   const double tau = (double)(a.t_next - a.count + i);  // re-indexed position of entry i
   for (int k = threadIdx.x; k < a.pairs; k += blockDim.x) s_cs[k] = rope_cos_sin(tau, a.omega[k]);
   __syncthreads();
@@ -680,7 +704,14 @@ __global__ void __launch_bounds__(256) rephase_kernel(const __grid_constant__ Re
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
       const int v = v0 + u * step;
-      if (v < nvec) raw[u] = __ldcs(reinterpret_cast<const uint4*>(src) + v);
+      if (v < nvec) {
+        if (kBoundsChecks && !bounds_ok(dev_range(a.cache, a.cache_bytes), reinterpret_cast<const uint4*>(src) + v,
+                                        sizeof(uint4), a.status)) {
+          raw[u] = make_uint4(0u, 0u, 0u, 0u);
+          continue;
+        }
+        raw[u] = __ldcs(reinterpret_cast<const uint4*>(src) + v);
+      }
     }
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
@@ -694,6 +725,9 @@ __global__ void __launch_bounds__(256) rephase_kernel(const __grid_constant__ Re
         rope_rotate_vec<V::kN>(x, d / 2, a.pairs, s_cs);
         w = V::pack(x);
       }
+      if (kBoundsChecks &&
+          !bounds_ok(dev_range(a.cache, a.cache_bytes), reinterpret_cast<uint4*>(dst) + v, sizeof(uint4), a.status))
+        continue;
       reinterpret_cast<uint4*>(dst)[v] = w;
     }
   }
@@ -702,10 +736,12 @@ __global__ void __launch_bounds__(256) rephase_kernel(const __grid_constant__ Re
 }  // namespace
 
 cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* st, int count, long long t_next,
-                           cudaStream_t stream) {
+                           unsigned int* status, cudaStream_t stream) {
   if (count <= 0 || g.rope_pairs <= 0) return cudaSuccess;
   RephaseArgs a;
   a.cache = reinterpret_cast<char*>(cache_base);
+  a.cache_bytes = (size_t)g.L * g.layer_bytes;
+  a.status = status;
   a.st = st;
   a.H = g.H; a.M = g.M; a.N = g.N; a.D = g.D;
   a.count = count;

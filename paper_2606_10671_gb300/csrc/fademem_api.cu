@@ -311,7 +311,7 @@ FADEMEM_API fademem_status fademem_consolidate(fademem_t h, void* stream_) {
   }
   if (h->g.rope_pairs > 0) {
     // Keys for attention: every entry rotated to its re-indexed position.
-    cudaError_t e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, stream);
+    cudaError_t e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, h->status, stream);
     if (e != cudaSuccess) return cuda_fail(e, "launching the re-phase kernel");
     ++h->launches;
   }
@@ -348,7 +348,7 @@ static fademem_status attend_impl(fademem_t h, int layer, const void* Q, const v
   cudaError_t e;
   if (h->g.dtype == FADEMEM_F32) {
     e = launch_attend_f32(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, reinterpret_cast<const float*>(Q),
-                          reinterpret_cast<float*>(out), Lq, h->cfg.scale, stream);
+                          reinterpret_cast<float*>(out), Lq, h->cfg.scale, h->status, stream);
   } else {
     char msg[256] = "";
     e = launch_attend_bf16(h->g, Kc, Vc, Lk, Kcur, Vcur, ncur, Q, out, Lq, h->cfg.scale, h->status, stream, msg,
@@ -793,7 +793,7 @@ FADEMEM_API fademem_status fademem_import_state(fademem_t h, const void* host_bu
   h->frames = hd.frames;
   h->la_valid = false;
   if (h->g.rope_pairs > 0 && h->count > 0) {
-    e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, stream);
+    e = launch_rephase(h->g, h->cache, cur_state(h), h->count, h->frames, h->status, stream);
     if (e != cudaSuccess) return cuda_fail(e, "launching the re-phase kernel");
     ++h->launches;
     if ((e = cudaStreamSynchronize(stream)) != cudaSuccess) return cuda_fail(e, "rebuilding the attention keys");
@@ -820,5 +820,7 @@ FADEMEM_API void fademem_destroy(fademem_t h) {
 }
 
 FADEMEM_API const char* fademem_last_error(void) { return g_err; }
+
+FADEMEM_API uint32_t fademem_build_flags(void) { return kBoundsChecks ? FADEMEM_BUILD_DEBUG_BOUNDS : 0u; }
 
 }  // extern "C"

@@ -28,6 +28,48 @@ constexpr uint32_t kStatusPlanOverflow = FADEMEM_STATUS_PLAN_OVERFLOW;    // mer
 constexpr uint32_t kStatusNearTie = FADEMEM_STATUS_NEAR_TIE;
 constexpr size_t kNearTieFrameOffset = 24;  // after the status word and the two counters
 
+// Device bounds checks.  Built with -DFADEMEM_DEBUG_BOUNDS (build.py
+// --debug-bounds, libfademem_debug.so), every kernel checks each global-memory
+// access against the buffer it belongs to and each table index against its
+// array; an access that fails is skipped and recorded as kStatusBounds in the
+// status word.  In the release build kBoundsChecks is false and every check
+// compiles away.
+#ifdef FADEMEM_DEBUG_BOUNDS
+constexpr bool kBoundsChecks = true;
+#else
+constexpr bool kBoundsChecks = false;
+#endif
+constexpr uint32_t kStatusBounds = FADEMEM_STATUS_BOUNDS;
+
+// The byte range [lo, hi) of one device buffer.
+struct DevRange {
+  const char* lo;
+  const char* hi;
+};
+__host__ __device__ inline DevRange dev_range(const void* base, size_t bytes) {
+  const char* p = static_cast<const char*>(base);
+  return DevRange{p, p + bytes};
+}
+// True if [p, p + bytes) lies in r (no pointer arithmetic that could wrap).
+__host__ __device__ inline bool range_holds(const DevRange& r, const void* p, size_t bytes) {
+  const char* c = static_cast<const char*>(p);
+  return c >= r.lo && c <= r.hi && (size_t)(r.hi - c) >= bytes;
+}
+#ifdef __CUDACC__
+// True if [p, p + bytes) lies in r; otherwise records kStatusBounds.
+__device__ __forceinline__ bool bounds_ok(const DevRange& r, const void* p, size_t bytes, unsigned int* status) {
+  if (range_holds(r, p, bytes)) return true;
+  atomicOr(status, kStatusBounds);
+  return false;
+}
+// True if 0 <= i < n; otherwise records kStatusBounds.
+__device__ __forceinline__ bool index_ok(long long i, long long n, unsigned int* status) {
+  if (i >= 0 && i < n) return true;
+  atomicOr(status, kStatusBounds);
+  return false;
+}
+#endif
+
 // Entry table of the memory (Sec. 3.3 "memory entries"), temporal order.
 struct DevMeta {
   int count;
@@ -114,12 +156,12 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
 // entry table, K_att[slot_i] = stored K[slot_i] rotated to position
 // t_next - count + i (the rest of each row copied unchanged).
 cudaError_t launch_rephase(const Geometry& g, void* cache_base, const DevState* st, int count, long long t_next,
-                           cudaStream_t stream);
+                           unsigned int* status, cudaStream_t stream);
 // Attention over Lk memory keys (Kc/Vc: one layer's [H][M][N][D] memory) followed
 // by Lk2 current-chunk keys (Kcur/Vcur: [Lk2][H][D]); either count may be 0.
 cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
                               const void* Vcur, int Lk2, const float* Q, float* out, int Lq, float scale,
-                              cudaStream_t stream);
+                              unsigned int* status, cudaStream_t stream);
 // Returns cudaErrorNotSupported if the shape is outside the tensor-core path.
 cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
                                const void* Vcur, int Lk2, const void* Q, void* out, int Lq, float scale,

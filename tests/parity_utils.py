@@ -138,6 +138,11 @@ class Pair:
         self.rounds = new
 
     def check_entries(self):
+        """The entry table bit-exact against the oracle, and the device status word clear (no
+        time-out, count mismatch, plan overflow, uncertified decision or, in the bounds-checking
+        build, bounds failure); reading the word clears it."""
+        st, word = self.gpu.device_status(raise_on_error=False)
+        assert word == 0, f"device status 0x{word:x}"
         slot, first, span, mu2 = self.gpu.entries()
         o_slot, o_first, o_span, o_mu = self._ref().entries()
         assert slot.tolist() == o_slot.tolist(), (slot, o_slot)

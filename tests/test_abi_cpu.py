@@ -22,7 +22,7 @@ def _declared_symbols():
 def test_exports_every_declared_symbol(cuda_lib):
     lib = ctypes.CDLL(cuda_lib)
     declared = _declared_symbols()
-    assert len(declared) == 22
+    assert len(declared) == 23
     for name in declared:
         assert hasattr(lib, name), name
     assert sorted(capi.EXPORTS) == declared
@@ -33,6 +33,22 @@ def test_only_abi_symbols_exported(cuda_lib):
     out = subprocess.run(["nm", "-D", "--defined-only", cuda_lib], capture_output=True, text=True).stdout
     text = [ln.split()[-1] for ln in out.splitlines() if " T " in ln]
     assert sorted(text) == _declared_symbols()
+
+
+def test_build_flags(cuda_lib):
+    """The release library reports no build flags.  The bounds-checking build (nvcc,
+    -DFADEMEM_DEBUG_BOUNDS; compiled here, no GPU needed) reports FADEMEM_BUILD_DEBUG_BOUNDS
+    and exports exactly the same symbols."""
+    import subprocess
+    from paper_2606_10671_gb300 import build
+    if not os.environ.get("FADEMEM_CUDA_LIB"):
+        assert ctypes.CDLL(cuda_lib).fademem_build_flags() == 0
+    debug = build.build_library(debug_bounds=True)
+    lib = ctypes.CDLL(debug)
+    lib.fademem_build_flags.restype = ctypes.c_uint32
+    assert lib.fademem_build_flags() == capi.BUILD_DEBUG_BOUNDS
+    out = subprocess.run(["nm", "-D", "--defined-only", debug], capture_output=True, text=True).stdout
+    assert sorted(ln.split()[-1] for ln in out.splitlines() if " T " in ln) == _declared_symbols()
 
 
 def _cfg(**kw):
