@@ -1,67 +1,365 @@
 // fp32 attention of query tokens over the memory (Sec. 3.3 last paragraph:
 // the memory is the cached context the backbone's attention sees).
-// Exact-precision path for the fp32 storage dtype: one warp per (query, head),
-// lanes split the head dimension, online softmax over every cached key in
-// fp32 (tf32 tensor cores would not meet a 1e-5 relative tolerance).
+// Exact-precision path for the fp32 storage dtype: fp32 FMAs throughout (tf32
+// tensor cores would not meet a 1e-5 relative tolerance), online softmax in
+// the exp2 domain.
+//
+// One block of 128 threads computes a tile of 32 queries of one head.  Tiles
+// of 32 keys are staged in shared memory by cp.async, double-buffered (the
+// next tile loads while this one is used).  Per tile:
+//   scores:  thread t holds a 2 x 4 block of S (queries 2(t/8) + {0,1}, keys
+//            t%8 + 8i), dot products over the head dimension from
+//            shared-memory float4 reads (conflict-free: padded rows);
+//            the 8 threads of a query pair reduce its row maximum and sum
+//            with three shuffles and write P (transposed) and the rescale
+//            factor to shared memory;
+//   P V:     thread t holds a 4 x (D/16) block of O (queries 4(t/16) + r,
+//            dims 4(t%16) + 64c), rescales it and adds the tile's P V.
+// The epilogue divides by the row sums.  When the query tiles are too few to
+// fill the GPU (small models), the keys of a tile are split over a cluster of
+// up to 8 blocks: each block runs the loop above over its share of the key
+// tiles, keeps its unnormalised O and its row maxima and sums in shared
+// memory, and after a cluster barrier each block combines a slice of the rows
+// from every block's partials through distributed shared memory (no global
+// scratch).
 #include <math.h>
 
 #include "fademem_internal.h"
+#include "per_device.h"
 
 namespace fademem {
 namespace {
 
+constexpr int kF32Threads = 128;
+constexpr int kBQ = 32;          // queries per block
+constexpr int kBK = 32;          // keys per tile
+constexpr int kPLD = kBQ + 4;    // row stride of the transposed P tile (floats)
+
+template <int D>
+struct F32Smem {
+  static constexpr int LD = D + 4;                     // padded row stride of Q and K (floats)
+  static constexpr int kQ = 0;                         // [kBQ][LD]
+  static constexpr int kK = kQ + kBQ * LD;             // [2][kBK][LD]
+  static constexpr int kV = kK + 2 * kBK * LD;         // [2][kBK][D]
+  static constexpr int kP = kV + 2 * kBK * D;          // [kBK][kPLD]: P transposed
+  static constexpr int kA = kP + kBK * kPLD;           // [kBQ]: rescale factor, then row sums
+  static constexpr int kFloats = kA + kBQ;
+  static constexpr size_t kBytes = (size_t)kFloats * 4;
+};
+
+// 16-byte global -> shared copy that bypasses registers (zero fill if !valid;
+// src must still be a valid address).
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
+
+// Shared-memory address of the same variable in block `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+               : "=r"(r)
+               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_cluster(uint32_t a) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_cluster4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(a)
+               : "memory");
+  return v;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ float dot4(const float4& a, const float4& b, float acc) {
+  acc = fmaf(a.x, b.x, acc);
+  acc = fmaf(a.y, b.y, acc);
+  acc = fmaf(a.z, b.z, acc);
+  return fmaf(a.w, b.w, acc);
+}
+
 // Keys: the Lk memory tokens of head h ([Lk][D] at Kc + h * head_stride), then
 // the Lk2 current-chunk tokens ([Lk2][H][D] at Kcur).
 template <int D>
-__global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict__ Kc, const float* __restrict__ Vc,
-                                                         int Lk, const float* __restrict__ Kcur,
-                                                         const float* __restrict__ Vcur, int Lk2,
-                                                         const float* __restrict__ Q, float* __restrict__ out,
-                                                         int Lq, int H, size_t head_stride, float scale_log2,
-                                                         unsigned int* status) {
-  constexpr int P = D / 32;
-  const int lane = threadIdx.x & 31;
-  const long long gw = (long long)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (gw >= (long long)Lq * H) return;
-  const int q = (int)(gw / H), h = (int)(gw % H);
-  const float* qp = Q + ((size_t)q * H + h) * D;
+__global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
+    const float* __restrict__ Kc, const float* __restrict__ Vc, int Lk, const float* __restrict__ Kcur,
+    const float* __restrict__ Vcur, int Lk2, const float* __restrict__ Q, float* __restrict__ out, int Lq, int H,
+    size_t head_stride, float scale_log2, int csplit, unsigned int* status) {
+  using S = F32Smem<D>;
+  constexpr int LD = S::LD;
+  constexpr int NC = D / 64;  // float4 columns of O per thread and query, 64 dims apart
+  extern __shared__ float4 smem4[];
+  float* sm = reinterpret_cast<float*>(smem4);
+  float* sQ = sm + S::kQ;
+  float* sK = sm + S::kK;
+  float* sV = sm + S::kV;
+  float* sP = sm + S::kP;
+  float* sA = sm + S::kA;
+  const int t = threadIdx.x;
+  // Cluster of csplit blocks (launched with that cluster shape along x): block
+  // `rank` of query tile blockIdx.x / csplit takes key tiles [tb, te).
+  const int rank = (int)(blockIdx.x % (unsigned)csplit);
+  const int q0 = (int)(blockIdx.x / (unsigned)csplit) * kBQ, h = blockIdx.y;
+  const int Lt = Lk + Lk2;
+  const int n_tiles = (Lt + kBK - 1) / kBK;
+  const int kt_begin = (int)((long long)n_tiles * rank / csplit) * kBK;
+  const int kt_end = min(Lt, (int)((long long)n_tiles * (rank + 1) / csplit) * kBK);
   // Buffers for the bounds-checking build: the layer's K and V memory, the
   // chunk's K and V, Q and out.
   const DevRange k_r = dev_range(Kc, (size_t)H * head_stride * 4), v_r = dev_range(Vc, (size_t)H * head_stride * 4);
   const DevRange kc_r = dev_range(Kcur, (size_t)Lk2 * H * D * 4), vc_r = dev_range(Vcur, (size_t)Lk2 * H * D * 4);
   const DevRange q_r = dev_range(Q, (size_t)Lq * H * D * 4), o_r = dev_range(out, (size_t)Lq * H * D * 4);
-  if (kBoundsChecks && !bounds_ok(q_r, qp, D * 4, status)) return;
-  float qv[P], o[P];
-#pragma unroll
-  for (int i = 0; i < P; ++i) { qv[i] = qp[lane + 32 * i]; o[i] = 0.f; }
+
+  for (int i = t; i < kBQ * D / 4; i += kF32Threads) {
+    const int r = i / (D / 4), c = (i % (D / 4)) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float* src = Q + ((size_t)(q0 + r) * H + h) * D + c;
+    if (q0 + r < Lq && (!kBoundsChecks || bounds_ok(q_r, src, 16, status))) v = *reinterpret_cast<const float4*>(src);
+    *reinterpret_cast<float4*>(sQ + r * LD + c) = v;
+  }
+
+  const int qp = t >> 3, kg = t & 7;    // scores: queries 2qp, 2qp+1; keys kg + 8i
+  const int quad = t >> 4, g = t & 15;  // P V: queries 4quad + r; dims 4g + 64c
   const float* Kh = Kc + (size_t)h * head_stride;  // keys of head h: [Lk][D], slots 0..count-1 contiguous
   const float* Vh = Vc + (size_t)h * head_stride;
-  float m = -INFINITY, l = 0.f;
-  for (int k = 0; k < Lk + Lk2; ++k) {
-    const float* kr = k < Lk ? Kh + (size_t)k * D : Kcur + ((size_t)(k - Lk) * H + h) * D;
-    const float* vr = k < Lk ? Vh + (size_t)k * D : Vcur + ((size_t)(k - Lk) * H + h) * D;
-    if (kBoundsChecks &&
-        (!bounds_ok(k < Lk ? k_r : kc_r, kr, D * 4, status) || !bounds_ok(k < Lk ? v_r : vc_r, vr, D * 4, status)))
-      continue;
-    float dot = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[4][4 * NC];
 #pragma unroll
-    for (int i = 0; i < P; ++i) dot = fmaf(qv[i], kr[lane + 32 * i], dot);
+  for (int r = 0; r < 4; ++r)
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    const float s = dot * scale_log2;
-    const float m_new = fmaxf(m, s);
-    const float c = exp2f(m - m_new);
-    const float p = exp2f(s - m_new);
-    l = l * c + p;
+    for (int e = 0; e < 4 * NC; ++e) o[r][e] = 0.f;
+
+  // Stage key tile kt (keys kt .. kt + kBK - 1; past the last key: zeros) into buffer buf.
+  auto load_tile = [&](int kt, int buf) {
+    float* dK = sK + buf * kBK * LD;
+    float* dV = sV + buf * kBK * D;
+    for (int i = t; i < kBK * D / 4; i += kF32Threads) {
+      const int r = i / (D / 4), c = (i % (D / 4)) * 4;
+      const int key = kt + r;
+      bool ok = key < Lt;
+      const float* kp = Q;  // any valid address for a zero-filled copy
+      const float* vp = Q;
+      if (ok) {
+        kp = key < Lk ? Kh + (size_t)key * D + c : Kcur + ((size_t)(key - Lk) * H + h) * D + c;
+        vp = key < Lk ? Vh + (size_t)key * D + c : Vcur + ((size_t)(key - Lk) * H + h) * D + c;
+        if (kBoundsChecks && !(bounds_ok(key < Lk ? k_r : kc_r, kp, 16, status) &&
+                               bounds_ok(key < Lk ? v_r : vc_r, vp, 16, status))) {
+          ok = false;
+          kp = vp = Q;
+        }
+      }
+      cp_async16(dK + r * LD + c, kp, ok);
+      cp_async16(dV + r * D + c, vp, ok);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+
+  if (kt_begin < kt_end) load_tile(kt_begin, 0);
+  for (int kt = kt_begin, it = 0; kt < kt_end; kt += kBK, ++it) {
+    // Every thread finished reading the other buffer (and P) in the previous
+    // iteration, so the next tile may load into it while this one is used.
+    if (kt + kBK < kt_end) {
+      load_tile(kt + kBK, (it + 1) & 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();  // this tile's copies (every thread's) have landed
+    const float* tK = sK + (it & 1) * kBK * LD;
+    const float* tV = sV + (it & 1) * kBK * D;
+
+    // ---- scores and the online softmax of rows 2qp, 2qp + 1 ----
+    float s[2][4];
 #pragma unroll
-    for (int i = 0; i < P; ++i) o[i] = fmaf(p, vr[lane + 32 * i], o[i] * c);
-    m = m_new;
+    for (int r = 0; r < 2; ++r)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) s[r][i] = 0.f;
+#pragma unroll 4
+    for (int d = 0; d < D; d += 4) {
+      const float4 qa = *reinterpret_cast<const float4*>(sQ + (2 * qp) * LD + d);
+      const float4 qb = *reinterpret_cast<const float4*>(sQ + (2 * qp + 1) * LD + d);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float4 k = *reinterpret_cast<const float4*>(tK + (kg + 8 * i) * LD + d);
+        s[0][i] = dot4(qa, k, s[0][i]);
+        s[1][i] = dot4(qb, k, s[1][i]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        s[r][i] = kt + kg + 8 * i < Lt ? s[r][i] * scale_log2 : -INFINITY;
+        mx = fmaxf(mx, s[r][i]);
+      }
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+      const float m_new = fmaxf(m_run[r], mx);  // finite: every tile holds a key
+      const float alpha = exp2f(m_run[r] - m_new);
+      float sum = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float p = exp2f(s[r][i] - m_new);
+        sum += p;
+        sP[(kg + 8 * i) * kPLD + 2 * qp + r] = p;
+      }
+      sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+      sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+      sum += __shfl_xor_sync(0xffffffffu, sum, 4);
+      l_run[r] = l_run[r] * alpha + sum;
+      m_run[r] = m_new;
+      if (kg == 0) sA[2 * qp + r] = alpha;
+    }
+    __syncthreads();
+
+    // ---- O <- alpha O + P V for rows 4quad .. 4quad + 3 ----
+    const float4 al = *reinterpret_cast<const float4*>(sA + 4 * quad);
+    const float alr[4] = {al.x, al.y, al.z, al.w};
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int e = 0; e < 4 * NC; ++e) o[r][e] *= alr[r];
+#pragma unroll 4
+    for (int k = 0; k < kBK; ++k) {
+      const float4 p4 = *reinterpret_cast<const float4*>(sP + k * kPLD + 4 * quad);
+      const float pr[4] = {p4.x, p4.y, p4.z, p4.w};
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        const float4 v = *reinterpret_cast<const float4*>(tV + k * D + 64 * c + 4 * g);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          o[r][4 * c + 0] = fmaf(pr[r], v.x, o[r][4 * c + 0]);
+          o[r][4 * c + 1] = fmaf(pr[r], v.y, o[r][4 * c + 1]);
+          o[r][4 * c + 2] = fmaf(pr[r], v.z, o[r][4 * c + 2]);
+          o[r][4 * c + 3] = fmaf(pr[r], v.w, o[r][4 * c + 3]);
+        }
+      }
+    }
+    __syncthreads();  // P, the rescale factors and this buffer are free again
   }
-  float* op = out + ((size_t)q * H + h) * D;
-  if (kBoundsChecks && !bounds_ok(o_r, op, D * 4, status)) return;
-  const float inv = 1.f / l;
+
+  if (csplit == 1) {
+    if (kg == 0) {
+      sA[2 * qp] = l_run[0];
+      sA[2 * qp + 1] = l_run[1];
+    }
+    __syncthreads();
 #pragma unroll
-  for (int i = 0; i < P; ++i) op[lane + 32 * i] = o[i] * inv;
+    for (int r = 0; r < 4; ++r) {
+      const int q = q0 + 4 * quad + r;
+      if (q >= Lq) continue;
+      const float inv = 1.f / sA[4 * quad + r];
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        float* dst = out + ((size_t)q * H + h) * D + 64 * c + 4 * g;
+        if (kBoundsChecks && !bounds_ok(o_r, dst, 16, status)) continue;
+        *reinterpret_cast<float4*>(dst) =
+            make_float4(o[r][4 * c] * inv, o[r][4 * c + 1] * inv, o[r][4 * c + 2] * inv, o[r][4 * c + 3] * inv);
+      }
+    }
+    return;
+  }
+
+  // ---- split keys: combine the cluster's partials ----
+  // This block's partials: unnormalised O [kBQ][D] over the K buffers, row
+  // maxima and sums (exp2 domain, this block's reference) over the P tile.
+  float* pO = sK;
+  float* pM = sP;
+  float* pL = sP + kBQ;
+  if (kg == 0) {
+    pM[2 * qp] = m_run[0];
+    pM[2 * qp + 1] = m_run[1];
+    pL[2 * qp] = l_run[0];
+    pL[2 * qp + 1] = l_run[1];
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+#pragma unroll
+    for (int c = 0; c < NC; ++c)
+      *reinterpret_cast<float4*>(pO + (4 * quad + r) * D + 64 * c + 4 * g) =
+          make_float4(o[r][4 * c], o[r][4 * c + 1], o[r][4 * c + 2], o[r][4 * c + 3]);
+  cluster_sync();  // every block's partials are written and visible to the cluster
+  // Block `rank` writes rows [rank * rows, (rank + 1) * rows) of the tile:
+  // out = sum_b 2^(m_b - M) O_b / sum_b 2^(m_b - M) l_b with M = max_b m_b.
+  const int rows = kBQ / csplit;
+  for (int i = t; i < rows * D / 4; i += kF32Threads) {
+    const int row = rank * rows + i / (D / 4), c = (i % (D / 4)) * 4;
+    float M = -INFINITY;
+    for (int b = 0; b < csplit; ++b) M = fmaxf(M, ld_cluster(cluster_addr(pM + row, b)));
+    float den = 0.f;
+    float4 num = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int b = 0; b < csplit; ++b) {
+      const float w = exp2f(ld_cluster(cluster_addr(pM + row, b)) - M);  // 0 for a block with no keys
+      den = fmaf(w, ld_cluster(cluster_addr(pL + row, b)), den);
+      const float4 ob = ld_cluster4(cluster_addr(pO + row * D + c, b));
+      num.x = fmaf(w, ob.x, num.x);
+      num.y = fmaf(w, ob.y, num.y);
+      num.z = fmaf(w, ob.z, num.z);
+      num.w = fmaf(w, ob.w, num.w);
+    }
+    const int q = q0 + row;
+    if (q >= Lq) continue;
+    float* dst = out + ((size_t)q * H + h) * D + c;
+    if (kBoundsChecks && !bounds_ok(o_r, dst, 16, status)) continue;
+    const float inv = 1.f / den;
+    *reinterpret_cast<float4*>(dst) = make_float4(num.x * inv, num.y * inv, num.z * inv, num.w * inv);
+  }
+  cluster_sync();  // no block leaves while another still reads its shared memory
+}
+
+template <int D>
+cudaError_t launch_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur, const void* Vcur,
+                       int Lk2, const float* Q, float* out, int Lq, float scale_log2, unsigned int* status,
+                       cudaStream_t stream) {
+  constexpr size_t smem = F32Smem<D>::kBytes;
+  if (smem > 48 * 1024) {
+    // The shared-memory opt-in is a per-device setting: once per device, with it current.
+    static PerDevice<char> opt_in;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    char done = 0;
+    if (!opt_in.get(dev, [&e](int, char* v) {
+          e = cudaFuncSetAttribute(attend_f32_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+          *v = 1;
+          return e == cudaSuccess;
+        }, &done))
+      return e != cudaSuccess ? e : cudaErrorInvalidDevice;
+  }
+  // Split the keys over a cluster of csplit blocks while the grid is far from
+  // filling the GPU (one wave at the kernel's occupancy) and each block keeps
+  // at least two key tiles.
+  const long long tiles_q = (Lq + kBQ - 1) / kBQ;
+  const long long blocks = tiles_q * g.H;
+  const int n_tiles = (Lk + Lk2 + kBK - 1) / kBK;
+  const long long wave = (long long)current_device_sm_count(148) * (smem > 64 * 1024 ? 2 : 4);
+  int csplit = 1;
+  while (csplit < 8 && blocks * csplit * 2 <= wave && n_tiles >= 4 * csplit) csplit *= 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(tiles_q * csplit), (unsigned)g.H);
+  cfg.blockDim = dim3(kF32Threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)csplit;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, attend_f32_kernel<D>, (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur,
+                            (const float*)Vcur, Lk2, Q, out, Lq, g.H, (size_t)g.M * g.N * g.D, scale_log2, csplit,
+                            status);
 }
 
 }  // namespace
@@ -69,20 +367,9 @@ __global__ void __launch_bounds__(256) attend_f32_kernel(const float* __restrict
 cudaError_t launch_attend_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk, const void* Kcur,
                               const void* Vcur, int Lk2, const float* Q, float* out, int Lq, float scale,
                               unsigned int* status, cudaStream_t stream) {
-  const long long warps = (long long)Lq * g.H;
-  const int threads = 256;
-  const long long blocks = (warps * 32 + threads - 1) / threads;
   const float scale_log2 = scale * 1.4426950408889634f;
-  const size_t head_stride = (size_t)g.M * g.N * g.D;
-  if (g.D == 128)
-    attend_f32_kernel<128><<<(unsigned)blocks, threads, 0, stream>>>(
-        (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
-        head_stride, scale_log2, status);
-  else
-    attend_f32_kernel<64><<<(unsigned)blocks, threads, 0, stream>>>(
-        (const float*)Kc, (const float*)Vc, Lk, (const float*)Kcur, (const float*)Vcur, Lk2, Q, out, Lq, g.H,
-        head_stride, scale_log2, status);
-  return cudaGetLastError();
+  if (g.D == 128) return launch_f32<128>(g, Kc, Vc, Lk, Kcur, Vcur, Lk2, Q, out, Lq, scale_log2, status, stream);
+  return launch_f32<64>(g, Kc, Vc, Lk, Kcur, Vcur, Lk2, Q, out, Lq, scale_log2, status, stream);
 }
 
 }  // namespace fademem
