@@ -232,32 +232,58 @@ class RoundingDepth:
     the anchor have r = 0.  a: the largest |input| over the entry's own source frames,
     per coordinate.  Merges are convex and elementwise, so the exact block and every
     rounded intermediate lie within +-a, and |stored - exact| <= r (2^-8 + 2^-20) a.
+
+    e (when the exact new blocks are given, one pass per call): a tighter bound per
+    coordinate, built along the merge tree.  A pass writes each merged entry as
+    round_bf16(sum_k w_k stored_k) over its sources k (the older entries it covers
+    and the new frames in its span), with fp32 weights and fp32 FMAs.  With
+    stored_k = exact_k + err_k, |err_k| <= e_k, convex weights and x = |exact|:
+      before rounding:  |y - exact_new| <= E = max_k e_k + 2^-19 max_k (x_k + e_k)
+                        (2^-20 for the fp32 weights, 2^-20 for the FMA chain);
+      after rounding:   e_new = E + 2^-8 (x_new + E).
+    Each rounding then costs 2^-8 of the magnitude of the block it rounds, not of
+    the largest input, which is what makes deep merged entries checkable.
     """
 
     def __init__(self, anchor: bool = True):
         self.anchor = anchor
         self.r = {}
         self.a = {}
+        self.e = {}
+        self.x = {}
         self.anchor_a = None
 
-    def update(self, before, frames_before, fresh, after, passes: int = 1):
+    def update(self, before, frames_before, fresh, after, passes: int = 1, exact=None):
         """One consolidate call: `before`/`after` the (first, span) lists of the entries,
-        `fresh` {frame: |values|} of the frames it inserted, `passes` fused passes."""
+        `fresh` {frame: |values|} of the frames it inserted, `passes` fused passes,
+        `exact` {(first, span): |exact block|} of the entries it created (optional)."""
         if 0 in fresh:
             self.anchor_a = fresh[0]
         old = set(before)
-        r, a = {}, {}
+        r, a, e, x = {}, {}, {}, {}
         for key in after:
             f, s = key
             if key in old:
                 r[key], a[key] = self.r[key], self.a[key]
+                if key in self.e:
+                    e[key], x[key] = self.e[key], self.x[key]
             elif f == 0 and self.anchor:
                 r[key], a[key] = 0, self.anchor_a
+                e[key], x[key] = np.zeros_like(self.anchor_a), self.anchor_a
             elif s == 1 and f >= frames_before:
                 r[key], a[key] = 0, fresh[f]
+                e[key], x[key] = np.zeros_like(fresh[f]), fresh[f]
             else:
                 inner = [k for k in self.r if k[0] >= f and k[0] + k[1] <= f + s]
-                parts = [self.a[k] for k in inner] + [x for g, x in fresh.items() if f <= g < f + s]
+                new_frames = [v for g, v in fresh.items() if f <= g < f + s]
+                parts = [self.a[k] for k in inner] + new_frames
                 r[key] = passes + max([self.r[k] for k in inner], default=0)
                 a[key] = np.maximum.reduce(parts)
-        self.r, self.a = r, a
+                if exact is not None and passes == 1 and all(k in self.e for k in inner):
+                    zero = np.zeros_like(a[key])
+                    emax = np.maximum.reduce([self.e[k] for k in inner] + [zero])
+                    src = np.maximum.reduce([self.x[k] + self.e[k] for k in inner] + new_frames)
+                    pre = emax + 2.0 ** -19 * src
+                    x[key] = exact[key]
+                    e[key] = pre + BF16_U * (exact[key] + pre)
+        self.r, self.a, self.e, self.x = r, a, e, x
