@@ -419,18 +419,22 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
       }
       for (int j = 0; ok && j < n_tiles; ++j) {
         const int g = j & 1, sv = j % kVStages;
-        if (!mbar_wait(barat(bar0, BAR_PFULL + g), (j >> 1) & 1, abort_flag) ||
-            !mbar_wait(barat(bar0, BAR_VFULL + sv), (j / kVStages) & 1, abort_flag)) {
+        // K_{j+2} and V_j (usually loaded long before) are waited for first and
+        // P_j, the wait that blocks, last, so that the tile's 16 MMAs go out as
+        // one burst with no wait between P_j V_j and Q K_{j+2}^T.  Neither load
+        // waits for P_j: their slots are freed by the completion of S_{j-1}
+        // (Q K_{j-1}^T, and P_{j-3} V_{j-3} issued before it).
+        const int jn = j + 2;
+        const int sk = jn % kKStages;
+        if ((jn < n_tiles && !mbar_wait(barat(bar0, BAR_KFULL + sk), (jn / kKStages) & 1, abort_flag)) ||
+            !mbar_wait(barat(bar0, BAR_VFULL + sv), (j / kVStages) & 1, abort_flag) ||
+            !mbar_wait(barat(bar0, BAR_PFULL + g), (j >> 1) & 1, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
         issue_pv8(tmem + kColO + g * kHD, tmem + g * kBN, dV0 + sv * kStageStep, idesc_pv, j >= 2 ? 1u : 0u);
-        const int jn = j + 2;
         if (jn < n_tiles) {
-          const int sk = jn % kKStages;
-          if (!mbar_wait(barat(bar0, BAR_KFULL + sk), (jn / kKStages) & 1, abort_flag)) { ok = false; break; }
-          tc_fence_after();
           issue_qk8(tmem + g * kBN, dQ, dK0 + sk * kStageStep, idesc_qk);
           // Completes with P_j V_j and S_{j+2}: the group's next S, and (through it)
           // the release of V slot j%3 and K slot (j+2)%3.
