@@ -389,6 +389,11 @@ def run_cuda(args):
         "data": "synthetic (AR(1) K/V rho=0.9, N(0,1) Q; no model weights)",
         "config": main_config(ws),
         "gpu_launches": r["launches"],  # counted by the library
+        # What was measured against what: the digest of the library's sources (the build stamp; the
+        # GPU machine's copy has no git metadata) and the peak figures every fraction divides by.
+        "build": {"source_digest": _b._digest([])[:16], "library": os.path.basename(_b.LIB)},
+        "peaks": {"hbm_gbs": hbm_peak, "bf16_tflops": bf16_peak, "bf16_tflops_sustained": bf16_sustained,
+                  "sm_max_mhz": sm_mhz, "kind": peak_kind},
         "host_enqueue_us_per_step": round(statistics.median(host_us), 1),  # binding + ABI calls, GPU idle
         "roofline": _attention_obj(t_attn, flops, bf16_peak, f"{peak_kind} bf16 burst", bf16_sustained,
                                    _profiled_traffic("attend_tc_wan13b.md",
