@@ -460,13 +460,28 @@ def _measure_rope(args, sets, out, flush, stream, dev, cons_ms_plain, hbm_peak, 
                     "ncu duration is in profiles/"}
 
 
+CONFIG_NAMES = ("tiny_fp32", "wan13b_30layer_rollout", "stress_deep_hierarchy", "wan14b_layer")
+
+
+def _alu_peak():
+    """fp32 FMA peak derived from the unit counts: SMs x 128 lanes x 2 flop x the maximum SM clock."""
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    return sms * FP32_LANES_PER_SM * 2 * _peaks()[3] * 1e6 / 1e12
+
+
 def _measure_configs(args, dev, flush, stream, gpu_index, cpu):
-    """The other workloads of the method, each with its own clock record and roofline."""
+    """The other workloads of the method, each with its own clock record and roofline.
+    --configs selects some of them; `k3b_wan13b_2heads` alone times only the fp32 attention
+    at a size that fills the GPU (otherwise it is part of tiny_fp32)."""
+    want = set(CONFIG_NAMES) if args.configs == "all" else set(args.configs.split(","))
     out = {}
     for name, fn in (("tiny_fp32", _cfg_tiny), ("wan13b_30layer_rollout", _cfg_rollout30),
                      ("stress_deep_hierarchy", _cfg_stress), ("wan14b_layer", _cfg_wan14b)):
-        out[name] = fn(args, dev, flush, stream, gpu_index, cpu)
-        torch.cuda.empty_cache()
+        if name in want:
+            out[name] = fn(args, dev, flush, stream, gpu_index, cpu)
+            torch.cuda.empty_cache()
+    if "k3b_wan13b_2heads" in want and "tiny_fp32" not in want:
+        out["k3b_wan13b_2heads"] = _k3b_large(dev, stream, gpu_index, _alu_peak())
     return out
 
 
@@ -843,6 +858,9 @@ def main():
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-configs", action="store_true", help="time the headline workload only")
+    ap.add_argument("--configs", default="all",
+                    help="comma-separated other workloads to time: " + ",".join(CONFIG_NAMES) +
+                         ",k3b_wan13b_2heads (default: all)")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="wan1.3b")
     ap.add_argument("--rope-pairs", type=int, default=22,
                     help="also time the workload with temporal RoPE handling on this many pairs (0: skip)")
