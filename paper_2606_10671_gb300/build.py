@@ -48,7 +48,9 @@ def _digest(extra: list[str]) -> str:
             h.update(name.encode())
             with open(path, "rb") as fh:
                 h.update(fh.read())
-    h.update(" ".join(ARCH + NVCC_FLAGS + extra).encode())
+    # The flags without the include directory's absolute path, so that the same sources
+    # give the same digest on every machine.
+    h.update(" ".join(ARCH + [f for f in NVCC_FLAGS if f != INCLUDE] + extra).encode())
     return h.hexdigest()
 
 
