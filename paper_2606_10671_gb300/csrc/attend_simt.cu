@@ -4,17 +4,21 @@
 // tensor cores would not meet a 1e-5 relative tolerance), online softmax in
 // the exp2 domain.
 //
-// One block of 128 threads computes a tile of 32 queries of one head.  Tiles
+// One block of 128 threads computes a tile of 64 queries of one head.  Tiles
 // of 32 keys are staged in shared memory by cp.async, double-buffered (the
 // next tile loads while this one is used).  Per tile:
-//   scores:  thread t holds a 2 x 4 block of S (queries 2(t/8) + {0,1}, keys
+//   scores:  thread t holds a 4 x 4 block of S (queries t/8 + 16r, keys
 //            t%8 + 8i), dot products over the head dimension from
-//            shared-memory float4 reads (conflict-free: padded rows);
-//            the 8 threads of a query pair reduce its row maximum and sum
-//            with three shuffles and write P (transposed) and the rescale
+//            shared-memory float4 reads (conflict-free: padded rows, and the
+//            four query groups of a warp on consecutive rows);
+//            the 8 threads of a query group reduce each row's maximum and
+//            sum with three shuffles and write P (transposed) and the rescale
 //            factor to shared memory;
-//   P V:     thread t holds a 4 x (D/16) block of O (queries 4(t/16) + r,
+//   P V:     thread t holds an 8 x (D/16) block of O (queries 8(t/16) + r,
 //            dims 4(t%16) + 64c), rescales it and adds the tile's P V.
+// The shared-memory pipe bounds this loop (every 16-byte-per-thread load
+// costs 4 wavefronts), so the blocks are sized for reuse: 4 FMAs per loaded
+// float in P V, 2 in the scores.
 // The epilogue divides by the row sums.  When the query tiles are too few to
 // fill the GPU (small models), the keys of a tile are split over a cluster of
 // up to 8 blocks: each block runs the loop above over its share of the key
@@ -24,6 +28,8 @@
 // scratch).
 #include <math.h>
 
+#include <algorithm>
+
 #include "fademem_internal.h"
 #include "per_device.h"
 
@@ -31,7 +37,9 @@ namespace fademem {
 namespace {
 
 constexpr int kF32Threads = 128;
-constexpr int kBQ = 32;          // queries per block
+constexpr int kBQ = 64;          // queries per block
+constexpr int kQS = kBQ / 16;    // score rows per thread: 16 query groups of 8 threads
+constexpr int kQO = kBQ / 8;     // output rows per thread: 8 row groups of 16 threads
 constexpr int kBK = 32;          // keys per tile
 constexpr int kPLD = kBQ + 4;    // row stride of the transposed P tile (floats)
 
@@ -126,14 +134,19 @@ __global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
     *reinterpret_cast<float4*>(sQ + r * LD + c) = v;
   }
 
-  const int qp = t >> 3, kg = t & 7;    // scores: queries 2qp, 2qp+1; keys kg + 8i
-  const int quad = t >> 4, g = t & 15;  // P V: queries 4quad + r; dims 4g + 64c
+  const int qg = t >> 3, kg = t & 7;    // scores: queries qg + 16r; keys kg + 8i
+  const int qo = t >> 4, g = t & 15;    // P V: queries kQO qo + r; dims 4g + 64c
   const float* Kh = Kc + (size_t)h * head_stride;  // keys of head h: [Lk][D], slots 0..count-1 contiguous
   const float* Vh = Vc + (size_t)h * head_stride;
-  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  float o[4][4 * NC];
+  float m_run[kQS], l_run[kQS];
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
+  for (int r = 0; r < kQS; ++r) {
+    m_run[r] = -INFINITY;
+    l_run[r] = 0.f;
+  }
+  float o[kQO][4 * NC];
+#pragma unroll
+  for (int r = 0; r < kQO; ++r)
 #pragma unroll
     for (int e = 0; e < 4 * NC; ++e) o[r][e] = 0.f;
 
@@ -176,25 +189,26 @@ __global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
     const float* tK = sK + (it & 1) * kBK * LD;
     const float* tV = sV + (it & 1) * kBK * D;
 
-    // ---- scores and the online softmax of rows 2qp, 2qp + 1 ----
-    float s[2][4];
+    // ---- scores and the online softmax of rows qg + 16r ----
+    float s[kQS][4];
 #pragma unroll
-    for (int r = 0; r < 2; ++r)
+    for (int r = 0; r < kQS; ++r)
 #pragma unroll
       for (int i = 0; i < 4; ++i) s[r][i] = 0.f;
-#pragma unroll 4
+#pragma unroll 2
     for (int d = 0; d < D; d += 4) {
-      const float4 qa = *reinterpret_cast<const float4*>(sQ + (2 * qp) * LD + d);
-      const float4 qb = *reinterpret_cast<const float4*>(sQ + (2 * qp + 1) * LD + d);
+      float4 q[kQS], k[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 k = *reinterpret_cast<const float4*>(tK + (kg + 8 * i) * LD + d);
-        s[0][i] = dot4(qa, k, s[0][i]);
-        s[1][i] = dot4(qb, k, s[1][i]);
-      }
+      for (int r = 0; r < kQS; ++r) q[r] = *reinterpret_cast<const float4*>(sQ + (qg + 16 * r) * LD + d);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) k[i] = *reinterpret_cast<const float4*>(tK + (kg + 8 * i) * LD + d);
+#pragma unroll
+      for (int r = 0; r < kQS; ++r)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) s[r][i] = dot4(q[r], k[i], s[r][i]);
     }
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
+    for (int r = 0; r < kQS; ++r) {
       float mx = -INFINITY;
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -211,33 +225,47 @@ __global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
       for (int i = 0; i < 4; ++i) {
         const float p = exp2f(s[r][i] - m_new);
         sum += p;
-        sP[(kg + 8 * i) * kPLD + 2 * qp + r] = p;
+        sP[(kg + 8 * i) * kPLD + qg + 16 * r] = p;
       }
       sum += __shfl_xor_sync(0xffffffffu, sum, 1);
       sum += __shfl_xor_sync(0xffffffffu, sum, 2);
       sum += __shfl_xor_sync(0xffffffffu, sum, 4);
       l_run[r] = l_run[r] * alpha + sum;
       m_run[r] = m_new;
-      if (kg == 0) sA[2 * qp + r] = alpha;
+      if (kg == 0) sA[qg + 16 * r] = alpha;
     }
     __syncthreads();
 
-    // ---- O <- alpha O + P V for rows 4quad .. 4quad + 3 ----
-    const float4 al = *reinterpret_cast<const float4*>(sA + 4 * quad);
-    const float alr[4] = {al.x, al.y, al.z, al.w};
+    // ---- O <- alpha O + P V for rows kQO qo .. kQO qo + kQO - 1 ----
+    float alr[kQO];
 #pragma unroll
-    for (int r = 0; r < 4; ++r)
+    for (int r = 0; r < kQO; r += 4) {
+      const float4 al = *reinterpret_cast<const float4*>(sA + kQO * qo + r);
+      alr[r] = al.x;
+      alr[r + 1] = al.y;
+      alr[r + 2] = al.z;
+      alr[r + 3] = al.w;
+    }
+#pragma unroll
+    for (int r = 0; r < kQO; ++r)
 #pragma unroll
       for (int e = 0; e < 4 * NC; ++e) o[r][e] *= alr[r];
-#pragma unroll 4
+#pragma unroll 2
     for (int k = 0; k < kBK; ++k) {
-      const float4 p4 = *reinterpret_cast<const float4*>(sP + k * kPLD + 4 * quad);
-      const float pr[4] = {p4.x, p4.y, p4.z, p4.w};
+      float pr[kQO];
+#pragma unroll
+      for (int r = 0; r < kQO; r += 4) {
+        const float4 p4 = *reinterpret_cast<const float4*>(sP + k * kPLD + kQO * qo + r);
+        pr[r] = p4.x;
+        pr[r + 1] = p4.y;
+        pr[r + 2] = p4.z;
+        pr[r + 3] = p4.w;
+      }
 #pragma unroll
       for (int c = 0; c < NC; ++c) {
         const float4 v = *reinterpret_cast<const float4*>(tV + k * D + 64 * c + 4 * g);
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
+        for (int r = 0; r < kQO; ++r) {
           o[r][4 * c + 0] = fmaf(pr[r], v.x, o[r][4 * c + 0]);
           o[r][4 * c + 1] = fmaf(pr[r], v.y, o[r][4 * c + 1]);
           o[r][4 * c + 2] = fmaf(pr[r], v.z, o[r][4 * c + 2]);
@@ -250,15 +278,15 @@ __global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
 
   if (csplit == 1) {
     if (kg == 0) {
-      sA[2 * qp] = l_run[0];
-      sA[2 * qp + 1] = l_run[1];
+#pragma unroll
+      for (int r = 0; r < kQS; ++r) sA[qg + 16 * r] = l_run[r];
     }
     __syncthreads();
 #pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const int q = q0 + 4 * quad + r;
+    for (int r = 0; r < kQO; ++r) {
+      const int q = q0 + kQO * qo + r;
       if (q >= Lq) continue;
-      const float inv = 1.f / sA[4 * quad + r];
+      const float inv = 1.f / sA[kQO * qo + r];
 #pragma unroll
       for (int c = 0; c < NC; ++c) {
         float* dst = out + ((size_t)q * H + h) * D + 64 * c + 4 * g;
@@ -277,16 +305,17 @@ __global__ void __launch_bounds__(kF32Threads) attend_f32_kernel(
   float* pM = sP;
   float* pL = sP + kBQ;
   if (kg == 0) {
-    pM[2 * qp] = m_run[0];
-    pM[2 * qp + 1] = m_run[1];
-    pL[2 * qp] = l_run[0];
-    pL[2 * qp + 1] = l_run[1];
+#pragma unroll
+    for (int r = 0; r < kQS; ++r) {
+      pM[qg + 16 * r] = m_run[r];
+      pL[qg + 16 * r] = l_run[r];
+    }
   }
 #pragma unroll
-  for (int r = 0; r < 4; ++r)
+  for (int r = 0; r < kQO; ++r)
 #pragma unroll
     for (int c = 0; c < NC; ++c)
-      *reinterpret_cast<float4*>(pO + (4 * quad + r) * D + 64 * c + 4 * g) =
+      *reinterpret_cast<float4*>(pO + (kQO * qo + r) * D + 64 * c + 4 * g) =
           make_float4(o[r][4 * c], o[r][4 * c + 1], o[r][4 * c + 2], o[r][4 * c + 3]);
   cluster_sync();  // every block's partials are written and visible to the cluster
   // Block `rank` writes rows [rank * rows, (rank + 1) * rows) of the tile:
@@ -342,7 +371,9 @@ cudaError_t launch_f32(const Geometry& g, const void* Kc, const void* Vc, int Lk
   const long long tiles_q = (Lq + kBQ - 1) / kBQ;
   const long long blocks = tiles_q * g.H;
   const int n_tiles = (Lk + Lk2 + kBK - 1) / kBK;
-  const long long wave = (long long)current_device_sm_count(148) * (smem > 64 * 1024 ? 2 : 4);
+  // Resident blocks per SM by shared memory (each block also reserves 1 KB).
+  const long long per_sm = std::max(1, std::min(8, (int)(233472 / (smem + 1024))));
+  const long long wave = (long long)current_device_sm_count(148) * per_sm;
   int csplit = 1;
   while (csplit < 8 && blocks * csplit * 2 <= wave && n_tiles >= 4 * csplit) csplit *= 2;
   cudaLaunchConfig_t cfg = {};
