@@ -164,6 +164,47 @@ def test_minimum_budget_and_multilayer():
         p.check_attend(p.queries(20, layer=l), layer=l)
 
 
+@pytest.mark.parametrize("dtype,beta", [(torch.float32, 0.3), (torch.bfloat16, 1.0)])
+def test_largest_budget_and_pending_frames(dtype, beta):
+    """The limits of one memory: the largest budget (FADEMEM_MAX_BUDGET = 64, so 65 entries
+    right after an append and 63 eligible pairs: every warp loop of the schedule runs two
+    32-lane chunks and the candidate mask uses 63 of its 64 bits), filled by the most frames
+    one consolidate accepts (FADEMEM_MAX_PENDING = 64 in one insert call: 16 fused passes),
+    then steady 3-frame segments that merge.  beta = 1 makes ties everywhere (lowest index)."""
+    from paper_2606_10671_gb300 import capi
+    D = 128 if dtype == torch.bfloat16 else 64
+    p = Pair(capi.FADEMEM_MAX_BUDGET, 2, D, 8, beta=beta, dtype=dtype, seed=41)
+    p.step(capi.FADEMEM_MAX_PENDING)
+    assert p.gpu.counts() == (capi.FADEMEM_MAX_BUDGET, capi.FADEMEM_MAX_PENDING)
+    p.check_entries()
+    p.check_memory()
+    for seg in range(12):
+        p.step(3)
+        p.check_entries()
+        p.check_memory()
+    assert p.gpu.counts() == (capi.FADEMEM_MAX_BUDGET, capi.FADEMEM_MAX_PENDING + 36)
+    p.check_attend(p.queries(100, step=1))
+    p.gpu.device_status()
+
+
+def test_largest_layer_count():
+    """FADEMEM_MAX_LAYERS = 128 layers in one handle: one schedule and one consolidation
+    launch over 256 (layer, K|V) rows, the frame pointers of every layer in one pass.  The
+    entry table, and the memory and attention of the first and last layers, against the
+    oracle."""
+    from paper_2606_10671_gb300 import capi
+    L = capi.FADEMEM_MAX_LAYERS
+    p = Pair(4, 1, 64, 8, beta=0.3, dtype=torch.float32, layers=L, seed=43, oracle_layers=[0, L - 1])
+    for seg in range(5):
+        p.step(3)
+        p.check_entries()
+        for l in (0, L - 1):
+            p.check_memory(l)
+    for l in (0, L - 1):
+        p.check_attend(p.queries(20, layer=l), layer=l)
+    p.gpu.device_status()
+
+
 def test_status_codes_on_gpu():
     from paper_2606_10671_gb300 import capi
     p = Pair(4, 2, 128, 16, dtype=torch.bfloat16, seed=7)
