@@ -245,6 +245,11 @@ def fademem_destroy(h: int):
     load().fademem_destroy(ctypes.c_void_p(h))
 
 
+def fademem_build_flags() -> int:
+    """FADEMEM_BUILD_* bits of the loaded library (BUILD_DEBUG_BOUNDS: the bounds-checking build)."""
+    return int(load().fademem_build_flags())
+
+
 def fademem_last_error() -> str:
     m = load().fademem_last_error()
     return m.decode() if m else ""
