@@ -869,6 +869,10 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.configs != "all":
+        unknown = set(args.configs.split(",")) - set(CONFIG_NAMES) - {"k3b_wan13b_2heads"}
+        if unknown:
+            ap.error(f"--configs: unknown workload(s) {sorted(unknown)}")
     global H, WORKLOAD
     H, WORKLOAD = WORKLOADS[args.workload]
     if args.workload != "wan1.3b":
