@@ -437,6 +437,9 @@ constexpr int kConsThreads = 256;
 // Resident blocks per SM: 4 (64 registers) while the sources fit, 3 for 12
 // sources or with the RoPE rotation.
 __host__ __device__ constexpr int cons_blocks_per_sm(int ns_max, bool rope) { return ns_max <= 9 && !rope ? 4 : 3; }
+// Vectors a thread handles in a consolidation with more rows than one wave
+// holds (each row is then split into blocks of this many vectors a thread).
+constexpr int kConsShortIters = 4;
 
 template <typename T, bool kMax, int kNS, bool kRope>
 __global__ void __launch_bounds__(kConsThreads, cons_blocks_per_sm(kNS, kRope)) consolidate_kernel(
@@ -620,12 +623,18 @@ cudaError_t launch_consolidate(const Geometry& g, void* cache_base, const DevSta
   a.layer_elems = g.layer_bytes / g.elem;
   a.srcs = srcs;
   const int nvec = g.N * dv;
-  // One wave: (SMs x resident blocks) spread evenly over the layer*K|V*head rows;
-  // each thread then strides over its row's vectors.
+  // While the layer*K|V*head rows fit in one wave (SMs x resident blocks), that
+  // wave is spread evenly over them and each thread strides over its row's
+  // vectors.  More rows than that (a memory of many layers) would end in a
+  // partial wave of whole rows, too few blocks to keep HBM busy while they
+  // stream their rows (a 30-layer consolidation ran at 82% of the copy peak
+  // so); there each row is cut into short blocks of kConsShortIters vectors a
+  // thread, and the last of many short waves ends with the others (97%).
   const int num_sms = current_device_sm_count(148);
   const int nsb = frames <= 2 ? 0 : frames == 3 ? 1 : 2;  // sources <= 3F: 6, 9 or 12
   const int rows = g.L * 2 * g.H;
-  int bx = (num_sms * cons_blocks_per_sm(6 + 3 * nsb, rope.pairs > 0) - 1) / rows;  // - 1: the lookahead block
+  const int wave = num_sms * cons_blocks_per_sm(6 + 3 * nsb, rope.pairs > 0) - 1;  // - 1: the lookahead block
+  int bx = rows <= wave ? wave / rows : (nvec + kConsThreads * kConsShortIters - 1) / (kConsThreads * kConsShortIters);
   const int bx_max = (nvec + kConsThreads - 1) / kConsThreads;
   if (bx > bx_max) bx = bx_max;
   if (bx < 1) bx = 1;
