@@ -51,6 +51,10 @@ constexpr uint32_t kOffBar = kOffV + kVStages * kTileBytes;
 // Per-row (m, l) of both groups for the epilogue: reuses K stage 0, which no
 // MMA reads any more once the final drain has completed.
 constexpr uint32_t kOffML = kOffK;
+// Row stride (floats) of a split tile's partial O in shared memory: 4 floats of
+// padding keep the rows' 16-byte stores and loads on distinct banks.
+constexpr int kPOStride = kHD + 4;
+static_assert((kBM * kPOStride + 2 * kBM) * 4 <= kVStages * kTileBytes, "split partials fit the V ring");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;  // + alignment slack
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns: S_0 [0,128), S_1 [128,256) fp32 (P_g overwrites the first 64
@@ -70,6 +74,7 @@ struct AttnParams {
   CUtensorMap tmV2;
   __nv_bfloat16* out;
   int Lq, Lk, Lk2, H;
+  int csplit;  // CTAs (a cluster) sharing one query tile's key tiles: 1, 2, 4 or 8
   float scale_log2;
   unsigned int* status;
 };
@@ -283,22 +288,38 @@ __device__ __forceinline__ void issue_pv8(uint32_t tO, uint32_t tP, uint64_t dV,
     umma_bf16_ts(tO, tP + kk * 8, dV + (uint64_t)(kk * (2048 >> 4)), idesc, kk > 0 ? 1u : acc0);
 }
 
+// kSplit: the query tile's keys are split over a cluster of p.csplit CTAs.  The
+// whole-tile instance (kSplit = false) keeps none of the split's bookkeeping.
+template <bool kSplit>
 __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = sbase + kOffBar;
   float* s_ml = reinterpret_cast<float*>(smem + kOffML);  // [2 groups][2 (m, l)][128 rows]
+  // A split tile's partials for the cluster's combine, over the V ring (idle
+  // once every MMA has completed): O [128][kPOStride], then m [128] and l [128].
+  float* s_po = reinterpret_cast<float*>(smem + kOffV);
+  float* s_pm = s_po + kBM * kPOStride;
+  float* s_pl = s_pm + kBM;
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int q0 = blockIdx.x * kBM;
+  // A query tile's key tiles may be split over a cluster of p.csplit CTAs
+  // (launched with that cluster shape along x): CTA `rank` takes key tiles
+  // [tb, tb + n_tiles) of the n_all, and the cluster combines its partials.
+  const int csplit = kSplit ? p.csplit : 1;
+  const int rank = kSplit ? (int)(blockIdx.x % (unsigned)csplit) : 0;
+  const int q0 = kSplit ? (int)(blockIdx.x / (unsigned)csplit) * kBM : (int)blockIdx.x * kBM;
   const int h = blockIdx.y;
   if (kBoundsChecks && threadIdx.x == 0) index_ok(h, p.H, p.status);
   // Key tiles 0..n1-1 come from the memory, n1..n1+n2-1 from the current chunk.
   const int n1 = (p.Lk + kBN - 1) / kBN;
-  const int n_tiles = n1 + (p.Lk2 + kBN - 1) / kBN;
+  const int n_all = n1 + (p.Lk2 + kBN - 1) / kBN;
+  const int tb = kSplit ? n_all * rank / csplit : 0;
+  const int n_tiles = kSplit ? n_all * (rank + 1) / csplit - tb : n_all;  // this CTA's key tiles (>= 4 when split)
+  constexpr bool split = kSplit;
 
   if (threadIdx.x == 0) {
     s_abort = 0;
@@ -358,18 +379,19 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
           break;
         }
         const uint32_t sK = sbase + kOffK + s * kTileBytes;
-        if (kBoundsChecks && !index_ok(j < n1 ? (long long)j * kBN : (long long)(j - n1) * kBN, j < n1 ? p.Lk : p.Lk2,
+        const int t = tb + j;  // key tile
+        if (kBoundsChecks && !index_ok(t < n1 ? (long long)t * kBN : (long long)(t - n1) * kBN, t < n1 ? p.Lk : p.Lk2,
                                        p.status)) {
           *abort_flag = 1;  // stop the CTA: every role's waits give up on the abort flag
           break;
         }
         mbar_expect_tx(full, kTileBytes);
-        if (j < n1) {
-          tma_load_3d(sK, &p.tmK, full, 0, j * kBN, h);
-          tma_load_3d(sK + kHalfBytes, &p.tmK, full, 64, j * kBN, h);
+        if (t < n1) {
+          tma_load_3d(sK, &p.tmK, full, 0, t * kBN, h);
+          tma_load_3d(sK + kHalfBytes, &p.tmK, full, 64, t * kBN, h);
         } else {
-          tma_load_3d(sK, &p.tmK2, full, 0, h, (j - n1) * kBN);
-          tma_load_3d(sK + kHalfBytes, &p.tmK2, full, 64, h, (j - n1) * kBN);
+          tma_load_3d(sK, &p.tmK2, full, 0, h, (t - n1) * kBN);
+          tma_load_3d(sK + kHalfBytes, &p.tmK2, full, 64, h, (t - n1) * kBN);
         }
       }
     }
@@ -384,13 +406,14 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
           break;
         }
         const uint32_t sV = sbase + kOffV + s * kTileBytes;
+        const int t = tb + j;  // key tile
         mbar_expect_tx(full, kTileBytes);
-        if (j < n1) {
-          tma_load_3d(sV, &p.tmV, full, 0, j * kBN, h);
-          tma_load_3d(sV + kHalfBytes, &p.tmV, full, 64, j * kBN, h);
+        if (t < n1) {
+          tma_load_3d(sV, &p.tmV, full, 0, t * kBN, h);
+          tma_load_3d(sV + kHalfBytes, &p.tmV, full, 64, t * kBN, h);
         } else {
-          tma_load_3d(sV, &p.tmV2, full, 0, h, (j - n1) * kBN);
-          tma_load_3d(sV + kHalfBytes, &p.tmV2, full, 64, h, (j - n1) * kBN);
+          tma_load_3d(sV, &p.tmV2, full, 0, h, (t - n1) * kBN);
+          tma_load_3d(sV + kHalfBytes, &p.tmV2, full, 64, h, (t - n1) * kBN);
         }
       }
     }
@@ -464,7 +487,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         if (j >= 2) mbar_arrive(barat(bar0, BAR_VEMPTY + (j - 2) % kVStages));
       }
       tc_fence_after();
-      const int valid = j < n1 ? p.Lk - j * kBN : p.Lk2 - (j - n1) * kBN;  // keys of this tile
+      const int t = tb + j;  // key tile
+      const int valid = t < n1 ? p.Lk - t * kBN : p.Lk2 - (t - n1) * kBN;  // keys of this tile
       // Fast path: exponentials against the running reference maximum m_run,
       // with no max over the tile first.  Any reference keeps the softmax exact
       // (it cancels in O / l) as long as no exponential overflows, and the row
@@ -575,9 +599,16 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
         const float m = has1 ? fmaxf(m0, m1) : m0;
         const float f0 = ex2(m0 - m);
         const float f1 = has1 ? ex2(m1 - m) : 0.f;
-        const float inv = 1.f / (l0 * f0 + l1 * f1);
+        const float l = l0 * f0 + l1 * f1;
+        // A split tile keeps this CTA's O unnormalised (relative to m) for the
+        // cluster's combine; a whole tile is divided by l here.
+        const float inv = split ? 1.f : 1.f / l;
         const float a0 = f0 * inv, a1 = f1 * inv;
         const int q = q0 + row;
+        if (split && grp == 0) {
+          s_pm[row] = m;
+          s_pl[row] = l;
+        }
         __nv_bfloat16* orow = p.out + ((size_t)q * p.H + h) * kHD;
         const uint32_t tO0 = tmem + kColO + lane_off;
         const uint32_t tO1 = tmem + kColO + kHD + lane_off;
@@ -595,6 +626,12 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
 #pragma unroll
               for (int e = 0; e < 8; ++e)
                 o[e] = __uint_as_float(r0[i + e]) * a0 + (has1 ? __uint_as_float(r1[i + e]) * a1 : 0.f);
+              if (split) {
+                float4* dst = reinterpret_cast<float4*>(s_po + row * kPOStride + col + i);
+                dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+                dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+                continue;
+              }
               uint4 v;
               v.x = pack_bf16(o[0], o[1]);
               v.y = pack_bf16(o[2], o[3]);
@@ -615,6 +652,47 @@ __global__ void __launch_bounds__(kThreads, 1) attend_tc_kernel(const __grid_con
   if (warp == kWarpMma) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
+  if (split) {
+    // ---- split keys: combine the cluster's partials ----
+    // Every CTA of the cluster passes both barriers, whatever happened above.
+    cluster_sync();  // every CTA's partials are written and visible to the cluster
+    // CTA `rank` writes rows [rank * rows, (rank + 1) * rows) of the tile:
+    // out = sum_b 2^(m_b - M) O_b / sum_b 2^(m_b - M) l_b with M = max_b m_b.
+    const int rows = kBM / csplit;
+    for (int i = threadIdx.x; i < rows * (kHD / 8); i += kThreads) {
+      const int row = rank * rows + i / (kHD / 8), c = (i % (kHD / 8)) * 8;
+      const int q = q0 + row;
+      if (q >= p.Lq) continue;
+      float M = -INFINITY;
+      for (int b = 0; b < csplit; ++b) M = fmaxf(M, ld_cluster(cluster_addr(s_pm + row, b)));
+      float den = 0.f;
+      float num[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      for (int b = 0; b < csplit; ++b) {
+        const float w = ex2(ld_cluster(cluster_addr(s_pm + row, b)) - M);
+        den = fmaf(w, ld_cluster(cluster_addr(s_pl + row, b)), den);
+        const uint32_t src = cluster_addr(s_po + row * kPOStride + c, b);
+        const float4 u0 = ld_cluster4(src), u1 = ld_cluster4(src + 16);
+        num[0] = fmaf(w, u0.x, num[0]);
+        num[1] = fmaf(w, u0.y, num[1]);
+        num[2] = fmaf(w, u0.z, num[2]);
+        num[3] = fmaf(w, u0.w, num[3]);
+        num[4] = fmaf(w, u1.x, num[4]);
+        num[5] = fmaf(w, u1.y, num[5]);
+        num[6] = fmaf(w, u1.z, num[6]);
+        num[7] = fmaf(w, u1.w, num[7]);
+      }
+      const float inv = 1.f / den;
+      uint4 v;
+      v.x = pack_bf16(num[0] * inv, num[1] * inv);
+      v.y = pack_bf16(num[2] * inv, num[3] * inv);
+      v.z = pack_bf16(num[4] * inv, num[5] * inv);
+      v.w = pack_bf16(num[6] * inv, num[7] * inv);
+      __nv_bfloat16* dst = p.out + ((size_t)q * p.H + h) * kHD + c;
+      if (!kBoundsChecks || bounds_ok(dev_range(p.out, (size_t)p.Lq * p.H * kHD * 2), dst, sizeof(uint4), p.status))
+        *reinterpret_cast<uint4*>(dst) = v;
+    }
+    cluster_sync();  // no CTA leaves while another still reads its shared memory
   }
 }
 
@@ -691,7 +769,9 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
     if (e != cudaSuccess) return e;
     char done = 0;
     if (!smem_opt_in.get(dev, [&e](int, char* v) {
-          e = cudaFuncSetAttribute(attend_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+          e = cudaFuncSetAttribute(attend_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+          if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(attend_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
           *v = 1;
           return e == cudaSuccess;
         }, &done))
@@ -719,17 +799,33 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
   prm.H = g.H;
   prm.scale_log2 = scale * 1.4426950408889634f;
   prm.status = status;
+  // One CTA per SM.  While the query tiles fill less than half the SMs (few
+  // queries, or few heads), split each tile's keys over a cluster of 2, 4 or 8
+  // CTAs (each keeping at least 4 key tiles), which combine their partials
+  // through distributed shared memory.
+  const long long tiles_q = (Lq + kBM - 1) / kBM;
+  const long long ctas = tiles_q * g.H;
+  const int n_all = (Lk + kBN - 1) / kBN + (Lk2 + kBN - 1) / kBN;
+  const long long sms = current_device_sm_count(148);
+  int csplit = 1;
+  while (csplit < 8 && ctas * csplit * 2 <= sms && n_all >= 4 * csplit) csplit *= 2;
+  prm.csplit = csplit;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((Lq + kBM - 1) / kBM, g.H);
+  cfg.gridDim = dim3((unsigned)(tiles_q * csplit), g.H);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmemBytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)csplit;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, attend_tc_kernel, prm);
+  cfg.numAttrs = csplit > 1 ? 2 : 1;
+  return csplit > 1 ? cudaLaunchKernelEx(&cfg, attend_tc_kernel<true>, prm)
+                    : cudaLaunchKernelEx(&cfg, attend_tc_kernel<false>, prm);
 }
 
 }  // namespace fademem

@@ -62,6 +62,34 @@ __device__ __forceinline__ bool bounds_ok(const DevRange& r, const void* p, size
   atomicOr(status, kStatusBounds);
   return false;
 }
+// Thread-block cluster helpers (distributed shared memory), for kernels that
+// split one tile's keys over a cluster and combine the partials.
+// Shared-memory address of the same variable in block `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+               : "=r"(r)
+               : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_cluster(uint32_t a) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_cluster4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(a)
+               : "memory");
+  return v;
+}
+// Every thread of every block of the cluster arrives (release) and waits
+// (acquire): shared-memory writes before it are visible cluster-wide after it.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
 // True if 0 <= i < n; otherwise records kStatusBounds.
 __device__ __forceinline__ bool index_ok(long long i, long long n, unsigned int* status) {
   if (i >= 0 && i < n) return true;

@@ -7,11 +7,12 @@ outputs) and each table index against its array; an access that fails is
 skipped and recorded as FADEMEM_STATUS_BOUNDS in the device status word, which
 the parity helpers read after every check of the entry table and the tests at
 their end, and which must stay clear.  This runs every test
-of test_gpu_parity.py and test_gpu_configs.py in a subprocess that loads that
-build: the seeded fuzz over every option, every consolidation kernel instance,
-RoPE, the current chunk, multi-layer memories up to 128 layers, the fp32 path,
-the full Wan-1.3B shapes, CUDA graphs, checkpoints, the attention's slow paths,
-the hour-long stress, the 30-layer rollout and the 40-layer Wan-14B memory.
+of test_gpu_parity.py, test_gpu_configs.py and test_gpu_attend_split.py in a
+subprocess that loads that build: the seeded fuzz over every option, every
+consolidation kernel instance, RoPE, the current chunk, multi-layer memories up
+to 128 layers, the fp32 path, the full Wan-1.3B shapes, CUDA graphs,
+checkpoints, the attention's slow paths and its cluster split, the hour-long
+stress, the 30-layer rollout and the 40-layer Wan-14B memory.
 They must pass unchanged, with the status word clear.
 """
 import ctypes
@@ -37,7 +38,8 @@ def test_parity_cases_under_bounds_checks():
     assert lib.fademem_build_flags() == capi.BUILD_DEBUG_BOUNDS
     env = dict(os.environ, FADEMEM_CUDA_LIB=debug)
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", "-m", "gpu",
-                        os.path.join(HERE, "test_gpu_parity.py"), os.path.join(HERE, "test_gpu_configs.py")],
+                        os.path.join(HERE, "test_gpu_parity.py"), os.path.join(HERE, "test_gpu_configs.py"),
+                        os.path.join(HERE, "test_gpu_attend_split.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=1500)
     tail = r.stdout[-3000:] + r.stderr[-2000:]
     assert r.returncode == 0, tail
