@@ -809,6 +809,38 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
   const long long sms = current_device_sm_count(148);
   int csplit = 1;
   while (csplit < 8 && ctas * csplit * 2 <= sms && n_all >= 4 * csplit) csplit *= 2;
+  // A cluster needs csplit SMs of one GPC with a CTA's shared memory free each:
+  // take the largest size the device can place (looked up once per device).
+  {
+    static PerDevice<int> max_cluster;
+    int dev = 0, fit = 1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    max_cluster.get(dev, [](int, int* v) {
+      *v = 1;
+      for (int c = 2; c <= 8; c *= 2) {
+        cudaLaunchConfig_t oc = {};
+        oc.gridDim = dim3((unsigned)c, 1);
+        oc.blockDim = dim3(kThreads);
+        oc.dynamicSmemBytes = kSmemBytes;
+        cudaLaunchAttribute ca[1];
+        ca[0].id = cudaLaunchAttributeClusterDimension;
+        ca[0].val.clusterDim.x = (unsigned)c;
+        ca[0].val.clusterDim.y = 1;
+        ca[0].val.clusterDim.z = 1;
+        oc.attrs = ca;
+        oc.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, attend_tc_kernel<true>, &oc) != cudaSuccess || n < 1) {
+          cudaGetLastError();  // clear a refused query; the smaller size stands
+          break;
+        }
+        *v = c;
+      }
+      return true;
+    }, &fit);
+    while (csplit > fit) csplit /= 2;
+  }
   prm.csplit = csplit;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(tiles_q * csplit), g.H);
