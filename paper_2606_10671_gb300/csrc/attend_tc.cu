@@ -22,6 +22,12 @@
 // so the tensor pipe and the exponential unit overlap.  The epilogue combines
 // (O_0, m_0, l_0) and (O_1, m_1, l_1) row by row.  Every mbarrier wait is
 // bounded; on time-out the CTA records it in the status word and leaves.
+//
+// When the tiles are too few to fill half the SMs, a tile's key tiles are
+// split over a thread-block cluster of 2, 4 or 8 CTAs (attend_tc_kernel<true>),
+// each running the pipeline above over its share and leaving its unnormalised
+// (O, m, l) in shared memory; after a cluster barrier each CTA assembles a
+// slice of the tile's rows from all of them through distributed shared memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <stdio.h>

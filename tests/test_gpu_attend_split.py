@@ -9,7 +9,8 @@ through distributed shared memory.  On a 152-SM GB300 these cases take:
   - 12 heads x 1 query tile over 49 key tiles (the Wan-1.3B head count, one
     128-query tile): clusters of 4;
   - one query, one head: clusters of 8, 127 of the tile's rows empty;
-  - memory keys and current-chunk keys in the same split (28 + 17 tiles);
+  - memory keys and current-chunk keys in the same split (28 + 17 tiles), and
+    the chunk's keys alone over an empty memory;
   - 3 heads x 3 query tiles (ragged, 300 queries) over 40 tiles: clusters of 8.
 Each is checked against the fp64 oracle, and the same call twice gives the same
 bytes (the combine adds the CTAs' partials in a fixed order).
@@ -56,6 +57,19 @@ def test_cluster_split_attention(name):
             a, b = p.gpu.attend(0, Q), p.gpu.attend(0, Q)
         torch.cuda.synchronize()
         assert torch.equal(a.view(torch.int16), b.view(torch.int16)), "the split attention is not deterministic"
+    st, word = p.gpu.device_status()
+    assert word == 0
+
+
+def test_cluster_split_over_the_chunk_alone():
+    """An empty memory: 128 queries of 2 heads attend over the 2100 current-chunk keys
+    alone (17 key tiles, clusters of 4 on 152 SMs), before and after the first segment."""
+    p = Pair(5, 2, 128, 700, beta=0.3, dtype=torch.bfloat16, seed=61)
+    Q = p.queries(128, step=0)
+    Kc, Vc = p.chunk(2100, step=0)
+    p.check_attend_ext(Q, Kc, Vc)
+    p.step(3)
+    p.check_attend_ext(Q, Kc, Vc)
     st, word = p.gpu.device_status()
     assert word == 0
 
