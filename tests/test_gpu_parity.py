@@ -205,6 +205,24 @@ def test_largest_layer_count():
     p.gpu.device_status()
 
 
+@pytest.mark.parametrize("dtype,D", [(torch.bfloat16, 128), (torch.float32, 64)])
+def test_consolidation_short_blocks_many_rows(dtype, D):
+    """More (layer, K|V, head) rows than one wave of consolidation blocks holds (64 layers
+    x 2 x 8 heads = 1024 rows against 607 on 152 SMs): each row is cut into short blocks
+    of 4 vectors a thread, here 2 blocks of 1024 and 576 vectors per row (100 tokens x 16
+    vectors).  Entry tables, the memory of three layers and attention against the oracle."""
+    L = 64
+    p = Pair(4, 8, D, 100, beta=0.3, dtype=dtype, layers=L, seed=47, oracle_layers=[0, 31, L - 1])
+    for seg in range(4):
+        p.step(3)
+        p.check_entries()
+        for l in (0, 31, L - 1):
+            p.check_memory(l)
+    p.check_attend(p.queries(130, layer=L - 1), layer=L - 1)
+    st, word = p.gpu.device_status()
+    assert word == 0
+
+
 def test_status_codes_on_gpu():
     from paper_2606_10671_gb300 import capi
     p = Pair(4, 2, 128, 16, dtype=torch.bfloat16, seed=7)
