@@ -49,13 +49,14 @@ class Pair:
 
     def __init__(self, budget, heads, head_dim, tokens, beta=0.3, anchor=True, op="weighted",
                  dtype=torch.bfloat16, layers=1, seed=0, rho=rho_const(0.9), tracked_heads=None, device_gen=False,
-                 oracle_layers=None, rope_pairs=0, rope_theta=10000.0):
+                 oracle_layers=None, rope_pairs=0, rope_theta=10000.0, scale=0.0):
         from paper_2606_10671_gb300 import FadeMem
         self.M, self.H, self.D, self.N, self.L = budget, heads, head_dim, tokens, layers
         self.dtype = dtype
         self.tracked = list(range(heads)) if tracked_heads is None else list(tracked_heads)
         self.gpu = FadeMem(budget, heads, head_dim, tokens, num_layers=layers, beta=beta, anchor=anchor, merge_op=op,
-                           dtype=dtype, rope_pairs=rope_pairs, rope_theta=rope_theta)
+                           dtype=dtype, rope_pairs=rope_pairs, rope_theta=rope_theta, scale=scale)
+        self.scale = None if scale == 0.0 else float(scale)  # the oracle's softmax scale (None: 1/sqrt(D))
         self.rope = rope_pairs > 0
         elems = tokens * len(self.tracked) * head_dim
         self.ora_layers = list(range(layers)) if oracle_layers is None else list(oracle_layers)
@@ -208,7 +209,7 @@ class Pair:
         Qt = Q.double().cpu().numpy()[:, self.tracked, :]
         Kc = Kcur.double().cpu().numpy()[:, self.tracked, :]
         Vc = Vcur.double().cpu().numpy()[:, self.tracked, :]
-        ref = self.ora[layer].attend_ext(Qt, Kc, Vc, self.N, len(self.tracked), self.D)
+        ref = self.ora[layer].attend_ext(Qt, Kc, Vc, self.N, len(self.tracked), self.D, scale=self.scale)
         return assert_close(out.double().cpu().numpy()[:, self.tracked, :], ref, self.dtype, "attention + chunk")
 
     def check_attend(self, Q: torch.Tensor, layer=0, rows=None):
@@ -220,7 +221,7 @@ class Pair:
         Qh = Q.double().cpu().numpy()
         og = out.double().cpu().numpy()
         Qt = Qh[:, self.tracked, :]
-        ref = self.ora[layer].attend(Qt, self.N, len(self.tracked), self.D)
+        ref = self.ora[layer].attend(Qt, self.N, len(self.tracked), self.D, scale=self.scale)
         return assert_close(og[:, self.tracked, :], ref, self.dtype, "attention")
 
 

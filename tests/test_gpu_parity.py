@@ -223,6 +223,28 @@ def test_consolidation_short_blocks_many_rows(dtype, D):
     assert word == 0
 
 
+@pytest.mark.parametrize("dtype,D,N,Lq,ncur,scale", [
+    (torch.bfloat16, 128, 100, 300, 0, 0.03),     # whole query tiles
+    (torch.bfloat16, 128, 1000, 128, 0, 0.25),    # keys split over a cluster
+    (torch.bfloat16, 128, 700, 200, 2100, 0.05),  # memory and chunk keys
+    (torch.float32, 64, 64, 192, 0, 0.4),         # the fp32 kernel
+])
+def test_configured_softmax_scale(dtype, D, N, Lq, ncur, scale):
+    """A softmax scale set in the configuration (not 1/sqrt(D)) reaches every attention
+    path: the oracle applies the same scale to q.k in fp64."""
+    p = Pair(5, 2, D, N, beta=0.3, dtype=dtype, seed=53, scale=scale)
+    for seg in range(2):
+        p.step(3)
+        Q = p.queries(Lq, step=seg)
+        if ncur:
+            Kc, Vc = p.chunk(ncur, step=seg)
+            p.check_attend_ext(Q, Kc, Vc)
+        else:
+            p.check_attend(Q)
+    st, word = p.gpu.device_status()
+    assert word == 0
+
+
 def test_status_codes_on_gpu():
     from paper_2606_10671_gb300 import capi
     p = Pair(4, 2, 128, 16, dtype=torch.bfloat16, seed=7)
