@@ -10,7 +10,7 @@ through distributed shared memory.  On a 152-SM GB300 these cases take:
     128-query tile): clusters of 4;
   - one query, one head: clusters of 8, 127 of the tile's rows empty;
   - memory keys and current-chunk keys in the same split (28 + 17 tiles), and
-    the chunk's keys alone over an empty memory;
+    the chunk's keys alone over an empty memory, and keys re-indexed by temporal RoPE;
   - 3 heads x 3 query tiles (ragged, 300 queries) over 40 tiles: clusters of 8.
 Each is checked against the fp64 oracle, and the same call twice gives the same
 bytes (the combine adds the CTAs' partials in a fixed order).
@@ -57,6 +57,17 @@ def test_cluster_split_attention(name):
             a, b = p.gpu.attend(0, Q), p.gpu.attend(0, Q)
         torch.cuda.synchronize()
         assert torch.equal(a.view(torch.int16), b.view(torch.int16)), "the split attention is not deterministic"
+    st, word = p.gpu.device_status()
+    assert word == 0
+
+
+def test_cluster_split_with_temporal_rope():
+    """Temporal RoPE (22 pairs): the split attends over the re-indexed keys, 2 heads x 1
+    query tile over 40 key tiles (clusters of 8)."""
+    p = Pair(5, 2, 128, 1000, beta=0.3, dtype=torch.bfloat16, seed=67, rope_pairs=22)
+    for seg in range(3):
+        p.step(3)
+        p.check_attend(p.queries(128, step=seg))
     st, word = p.gpu.device_status()
     assert word == 0
 
