@@ -472,7 +472,8 @@ def _alu_peak():
 def _measure_configs(args, dev, flush, stream, gpu_index, cpu):
     """The other workloads of the method, each with its own clock record and roofline.
     --configs selects some of them; `k3b_wan13b_2heads` alone times only the fp32 attention
-    at a size that fills the GPU (otherwise it is part of tiny_fp32)."""
+    at a size that fills the GPU (otherwise it is part of tiny_fp32), and `attend_128_queries`
+    the bf16 attention of one query tile per head (its keys split over a cluster)."""
     want = set(CONFIG_NAMES) if args.configs == "all" else set(args.configs.split(","))
     out = {}
     for name, fn in (("tiny_fp32", _cfg_tiny), ("wan13b_30layer_rollout", _cfg_rollout30),
@@ -482,6 +483,9 @@ def _measure_configs(args, dev, flush, stream, gpu_index, cpu):
             torch.cuda.empty_cache()
     if "k3b_wan13b_2heads" in want and "tiny_fp32" not in want:
         out["k3b_wan13b_2heads"] = _k3b_large(dev, stream, gpu_index, _alu_peak())
+    if args.configs == "all" or "attend_128_queries" in want:
+        out["attend_128_queries"] = _attend_few_queries(dev, flush, stream, gpu_index)
+        torch.cuda.empty_cache()
     return out
 
 
@@ -631,6 +635,54 @@ def _k3b_large(dev, stream, gpu_index, alu_peak):
     return {"ms_per_attend": round(statistics.median(ts), 3), "flops_per_attend": flops,
             "achieved": round(tf, 2), "peak": round(alu_peak, 1), "unit": "TFLOP/s", "frac": round(tf / alu_peak, 4),
             "bound": "alu", "clocks": clk.summary()}
+
+
+def _attend_few_queries(dev, flush, stream, gpu_index):
+    """The bf16 attention with too few query tiles to fill the GPU: one 128-query tile of each of
+    the 12 heads over the steady-state Wan-1.3B memory (32,760 keys per head).  The launcher
+    splits each tile's keys over a thread-block cluster (of 8 CTAs on 152 SMs: 96 CTAs).  L2
+    flushed before each attend."""
+    from paper_2606_10671_gb300 import FadeMem
+    from synth import device_queries
+    _, bf16_peak, _, _, peak_kind = _peaks()
+    mem = FadeMem(M, H, D, N, beta=BETA, anchor=True, dtype=torch.bfloat16, device=dev)
+    sets = _segment_inputs(2000, 2, dev)
+    for s in range(WARM_SEGMENTS):
+        K, V, _ = sets[s % 2]
+        mem.insert(0, K, V)
+        mem.consolidate()
+    lq = 128
+    Q = device_queries((lq, H, D), 2000, 0, 9, device=dev)
+    o = torch.empty((lq, H, D), dtype=torch.bfloat16, device=dev)
+    for _ in range(3):
+        mem.attend(0, Q, o)
+    torch.cuda.synchronize()
+    ev = []
+    with ClockSampler(gpu_index) as clk:
+        for _ in range(20):
+            flush()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            mem.attend(0, Q, o)
+            e1.record(stream)
+            ev.append((e0, e1))
+        torch.cuda.synchronize()
+    mem.device_status()
+    ts = [e0.elapsed_time(e1) for e0, e1 in ev]
+    hbm_peak = _peaks()[0]
+    # One query tile per head reads each head's keys and values once: 128 FLOP per byte, below
+    # the ridge (measured bf16 peak / HBM copy peak = 284), so HBM bounds this launch.
+    nbytes = 2 * M * N * H * D * 2 + 2 * lq * H * D * 2  # K and V of the memory, Q and out
+    gbs = nbytes / (statistics.mean(ts) / 1e3) / 1e9
+    return {"workload": "one 128-query tile x 12 heads over the steady-state Wan-1.3B memory (21 entries x "
+                        "1560 tokens); bf16; keys split over a thread-block cluster",
+            "attend": _attention_obj(ts, 4.0 * lq * M * N * H * D, bf16_peak, f"{peak_kind} bf16 burst"),
+            "roofline": {"bound": "hbm", "bytes_per_launch": nbytes, "achieved": round(gbs, 1), "peak": hbm_peak,
+                         "unit": "GB/s", "frac": round(gbs / hbm_peak, 4),
+                         "traffic": _profiled_traffic("attend_tc_split_wan13b_128q.md",
+                                                      "paper_2606_10671_gb300/csrc/attend_tc.cu"),
+                         "note": "128 FLOP per byte, below the ridge of 284: the memory's K and V read once"},
+            "clocks": clk.summary(), "l2": "flushed before every attend"}
 
 
 def _cfg_rollout30(args, dev, flush, stream, gpu_index, cpu):
@@ -860,7 +912,7 @@ def main():
     ap.add_argument("--no-configs", action="store_true", help="time the headline workload only")
     ap.add_argument("--configs", default="all",
                     help="comma-separated other workloads to time: " + ",".join(CONFIG_NAMES) +
-                         ",k3b_wan13b_2heads (default: all)")
+                         ",k3b_wan13b_2heads,attend_128_queries (default: all)")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="wan1.3b")
     ap.add_argument("--rope-pairs", type=int, default=22,
                     help="also time the workload with temporal RoPE handling on this many pairs (0: skip)")
@@ -870,7 +922,7 @@ def main():
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.configs != "all":
-        unknown = set(args.configs.split(",")) - set(CONFIG_NAMES) - {"k3b_wan13b_2heads"}
+        unknown = set(args.configs.split(",")) - set(CONFIG_NAMES) - {"k3b_wan13b_2heads", "attend_128_queries"}
         if unknown:
             ap.error(f"--configs: unknown workload(s) {sorted(unknown)}")
     global H, WORKLOAD

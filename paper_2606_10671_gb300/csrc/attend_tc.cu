@@ -814,7 +814,7 @@ cudaError_t launch_attend_bf16(const Geometry& g, const void* Kc, const void* Vc
   const int n_all = (Lk + kBN - 1) / kBN + (Lk2 + kBN - 1) / kBN;
   const long long sms = current_device_sm_count(148);
   int csplit = 1;
-  while (csplit < 8 && ctas * csplit * 2 <= sms && n_all >= 4 * csplit) csplit *= 2;
+  while (csplit < 8 && ctas * csplit * 2 <= sms && n_all >= 8 * csplit) csplit *= 2;
   // A cluster needs csplit SMs of one GPC with a CTA's shared memory free each:
   // take the largest size the device can place (looked up once per device).
   {

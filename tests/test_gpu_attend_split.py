@@ -7,7 +7,7 @@ after a cluster barrier, assembles a slice of the tile's rows from all of them
 through distributed shared memory.  On a 152-SM GB300 these cases take:
   - 2 heads x 1 query tile over 40 key tiles: clusters of 8;
   - 12 heads x 1 query tile over 49 key tiles (the Wan-1.3B head count, one
-    128-query tile): clusters of 4;
+    128-query tile): clusters of 8, 96 CTAs;
   - one query, one head: clusters of 8, 127 of the tile's rows empty;
   - memory keys and current-chunk keys in the same split (28 + 17 tiles), and
     the chunk's keys alone over an empty memory, and keys re-indexed by temporal RoPE;
@@ -74,7 +74,8 @@ def test_cluster_split_with_temporal_rope():
 
 def test_cluster_split_over_the_chunk_alone():
     """An empty memory: 128 queries of 2 heads attend over the 2100 current-chunk keys
-    alone (17 key tiles, clusters of 4 on 152 SMs), before and after the first segment."""
+    alone (17 key tiles, clusters of 4 on 152 SMs: at least 4 key tiles a CTA), then with the
+    first segment's 17 tiles of memory keys before them (34 tiles, clusters of 8)."""
     p = Pair(5, 2, 128, 700, beta=0.3, dtype=torch.bfloat16, seed=61)
     Q = p.queries(128, step=0)
     Kc, Vc = p.chunk(2100, step=0)
